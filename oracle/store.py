@@ -1,0 +1,179 @@
+"""Oracle of the parameter manager: intents, replicas, pull, push, sync.
+
+TEST INFRASTRUCTURE ONLY (see oracle/__init__.py).
+
+State follows the paper's description of AdaPM with worker slots in the role
+of nodes and replication always chosen (the paper's "AdaPM w/o relocation"
+variant, Sec. 5.5):
+
+  main[K][D]        the main copy of every parameter (fp32)
+  clock[w]          worker w's logical clock C^w, starts at 0 (Sec. 3)
+  intents[w]        recorded Intent(keys, C_start, C_end) calls of worker w
+  replicas[w][k]    (val[D], acc[D]) for every key with a replica at w;
+                    val is the worker's local copy, acc the updates it wrote
+                    since the replica was created or last refreshed
+
+Definitions
+  * An intent is active while C_start <= C^w < C_end, inactive before,
+    expired after (Sec. 3).  A key is in the active set A_w(c) when some
+    recorded intent of w containing it is active at c.  Keys inside one call
+    are a set: repeats count once.
+  * Replica lifetime (Sec. 4.1): a replica exists for exactly the span in
+    which the worker has active intent.  After every call R_w = A_w(C^w).
+    Replicas are destroyed before new ones are created, each in ascending
+    key order; a key that stays active keeps its replica untouched, which is
+    how one intent extends another (Sec. 3).
+  * Creating a replica copies main[k] and zeroes acc; destroying one merges
+    acc into main[k] (App. B.1.2: replica holders send their updates to the
+    owner).
+  * pull: a key with a replica at w reads the local copy; any other key reads
+    the main copy, which is always current (Sec. 5.1; intent is optional,
+    Sec. 4).
+  * push: the rows of each distinct key are summed in order of appearance and
+    added to both val and acc of w's replica, or to main when w holds none.
+  * sync: for every key with at least one replica, main[k] += sum over the
+    holders (ascending worker) of acc, then every holder's val = main[k] and
+    acc = 0 (App. B.1.2: the owner merges the updates and propagates them to
+    the replica holders; sending only unseen versions gives the same values).
+
+Arithmetic: every sum runs in fp64 and is rounded to fp32 once when stored.
+"""
+import numpy as np
+
+
+class OracleError(ValueError):
+    """An argument the parameter manager must reject (bad worker, key out of range)."""
+
+
+def _f32(x):
+    return np.asarray(x, dtype=np.float64).astype(np.float32)
+
+
+class ParameterManagerOracle:
+    def __init__(self, num_keys, value_len, num_workers, init):
+        init = np.asarray(init, dtype=np.float32)
+        if init.shape != (num_keys, value_len):
+            raise OracleError("init must have shape (num_keys, value_len)")
+        self.K = int(num_keys)
+        self.D = int(value_len)
+        self.W = int(num_workers)
+        self.main = init.copy()
+        self.clock = [0] * self.W
+        self.intents = [[] for _ in range(self.W)]   # entries: (frozenset keys, start, end)
+        self.replicas = [dict() for _ in range(self.W)]
+
+    # -- argument checks ---------------------------------------------------
+    def _check_worker(self, w):
+        if not (0 <= w < self.W):
+            raise OracleError(f"worker {w} out of range")
+
+    def _check_keys(self, keys):
+        keys = np.asarray(keys, dtype=np.int64).reshape(-1)
+        if keys.size and (keys.min() < 0 or keys.max() >= self.K):
+            raise OracleError("key out of range")
+        return keys
+
+    # -- intent windows (Sec. 3) --------------------------------------------
+    def _is_active(self, start, end, c):
+        return start <= c < end
+
+    def active_set(self, w, c=None):
+        c = self.clock[w] if c is None else c
+        out = set()
+        for keys, s, e in self.intents[w]:
+            if self._is_active(s, e, c):
+                out |= keys
+        return out
+
+    def refcount(self, w, k):
+        """Number of w's intent calls that are active now and contain k."""
+        c = self.clock[w]
+        return sum(1 for keys, s, e in self.intents[w] if self._is_active(s, e, c) and k in keys)
+
+    def _reconcile(self, w):
+        """Make R_w equal A_w(C^w): destroy, then create, each in ascending key order."""
+        active = self.active_set(w)
+        held = set(self.replicas[w])
+        for k in sorted(held - active):
+            val, acc = self.replicas[w].pop(k)
+            self.main[k] = _f32(self.main[k].astype(np.float64) + acc.astype(np.float64))
+        for k in sorted(active - held):
+            self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+        # expired intents can never become active again (clocks only rise)
+        c = self.clock[w]
+        self.intents[w] = [(keys, s, e) for keys, s, e in self.intents[w] if e > c]
+
+    def intent(self, w, keys, start, end):
+        """Intent(keys, C_start, C_end) of worker w; the optional type is not modelled."""
+        self._check_worker(w)
+        keys = self._check_keys(keys)
+        start, end = int(start), int(end)
+        if end <= start or end <= self.clock[w]:
+            return                      # empty or already expired window: nothing to do
+        self.intents[w].append((frozenset(int(k) for k in keys), start, end))
+        self._reconcile(w)              # activates now if start <= C^w
+
+    def advance_clock(self, w):
+        self._check_worker(w)
+        self.clock[w] += 1
+        self._reconcile(w)
+
+    # -- access ----------------------------------------------------------------
+    def pull(self, w, keys):
+        self._check_worker(w)
+        keys = self._check_keys(keys)
+        out = np.empty((keys.size, self.D), dtype=np.float32)
+        reps = self.replicas[w]
+        for i, k in enumerate(keys.tolist()):
+            out[i] = reps[k][0] if k in reps else self.main[k]
+        return out
+
+    def push(self, w, keys, deltas):
+        self._check_worker(w)
+        keys = self._check_keys(keys)
+        deltas = np.asarray(deltas, dtype=np.float32).reshape(keys.size, self.D)
+        groups = {}
+        for i, k in enumerate(keys.tolist()):
+            groups.setdefault(k, []).append(i)
+        reps = self.replicas[w]
+        for k in sorted(groups):
+            s = np.zeros(self.D, dtype=np.float64)
+            for i in groups[k]:                      # order of appearance
+                s += deltas[i].astype(np.float64)
+            if k in reps:
+                val, acc = reps[k]
+                reps[k] = (_f32(val.astype(np.float64) + s), _f32(acc.astype(np.float64) + s))
+            else:
+                self.main[k] = _f32(self.main[k].astype(np.float64) + s)
+
+    def sync(self):
+        keys = sorted(set().union(*[set(r) for r in self.replicas]))
+        for k in keys:
+            total = self.main[k].astype(np.float64)
+            holders = [w for w in range(self.W) if k in self.replicas[w]]
+            for w in holders:                        # ascending worker
+                total = total + self.replicas[w][k][1].astype(np.float64)
+            self.main[k] = _f32(total)
+            for w in holders:
+                self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+
+    # -- inspection --------------------------------------------------------------
+    def replica_keys(self, w):
+        self._check_worker(w)
+        return np.array(sorted(self.replicas[w]), dtype=np.int64)
+
+    def replica_values(self, w):
+        """(keys ascending, val rows, acc rows) of worker w's replicas."""
+        ks = self.replica_keys(w)
+        val = np.array([self.replicas[w][k][0] for k in ks.tolist()], dtype=np.float32).reshape(-1, self.D)
+        acc = np.array([self.replicas[w][k][1] for k in ks.tolist()], dtype=np.float32).reshape(-1, self.D)
+        return ks, val, acc
+
+    def refcounts(self, w, keys):
+        self._check_worker(w)
+        keys = self._check_keys(keys)
+        return np.array([self.refcount(w, int(k)) for k in keys], dtype=np.int64)
+
+    def read_main(self, keys):
+        keys = self._check_keys(keys)
+        return self.main[keys].copy()
