@@ -1,0 +1,203 @@
+/*
+ * adapm.h -- C ABI of a GB300 parameter manager driven by intent signals.
+ *
+ * Method: AdaPM, "Good Intentions: Adaptive Parameter Management via Intent
+ * Signaling" (arXiv 2206.00470).  Workers announce, through Intent(), which
+ * keys they will access in a window of their own logical clock (Sec. 3).  The
+ * manager keeps a replica of each such key at the worker for exactly the
+ * span of the intent (Sec. 4.1, selective replication; this library always
+ * replicates, the paper's "AdaPM w/o relocation" of Sec. 5.5), serves the
+ * worker's reads from the replica, accumulates the worker's writes in it, and
+ * merges the accumulated updates into the main copy when the replica is
+ * destroyed or when sync() runs (App. B.1.2).  Access without intent is
+ * allowed at any time and goes to the main copy (Sec. 4, "optional intent").
+ * W workers are worker slots that share one GPU.
+ *
+ * Conventions for every call
+ *   - Keys are uint32 in [0, num_keys).  Value rows are value_len fp32,
+ *     row-major, value_len a multiple of 4 (16-byte rows).
+ *   - Array arguments may be device pointers or host pointers (pinned or
+ *     pageable); the library detects which with cudaPointerGetAttributes.
+ *     Host inputs are copied to the device on the library stream; a host
+ *     output is filled by a device-to-host copy on the library stream.
+ *   - Calls are ordered on the library stream and return once their work is
+ *     enqueued.  Device and pinned host arrays are read and written in
+ *     stream order: keep inputs unchanged, and read outputs only, after
+ *     adapm_wait() (or a synchronisation of the stream).  Pageable host
+ *     inputs are copied before the call returns and may be reused at once.
+ *   - The caller owns every array it passes; the library owns all of its
+ *     device state and frees it in adapm_destroy().
+ *   - Argument errors (null context or pointer, worker >= num_workers,
+ *     n > 2^31) return ADAPM_EINVAL synchronously and change nothing.
+ *   - Errors found on the device are sticky and returned by adapm_wait():
+ *     ADAPM_ERANGE for a key >= num_keys (the element is skipped; a pulled
+ *     row for it is zero), ADAPM_ENOMEM when replica_capacity is exhausted
+ *     (the replicas of that call are not created and reads of those keys go
+ *     to the main copy), ADAPM_ESTATE for a refcount overflow (more than
+ *     65535 overlapping intents of one worker on one key).
+ *   - ADAPM_ECUDA reports a CUDA runtime error; the context is then unusable.
+ *   - No C++ exception crosses the ABI.  A context is driven by one host
+ *     thread at a time.
+ */
+#ifndef ADAPM_H
+#define ADAPM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ADAPM_OK = 0,
+  ADAPM_EINVAL = 1,
+  ADAPM_ERANGE = 2,
+  ADAPM_ENOMEM = 3,
+  ADAPM_ESTATE = 4,
+  ADAPM_ECUDA = 5,
+  ADAPM_ETIMEOUT = 6
+} adapm_status;
+
+typedef struct adapm_ctx adapm_ctx; /* opaque; created and freed by the library */
+
+typedef struct {
+  uint64_t num_keys;         /* K, 1 <= K < 2^32 - 1 */
+  uint32_t value_len;        /* D floats per key, multiple of 4, <= 1024 */
+  uint32_t num_workers;      /* W, 1 <= W <= 32 */
+  uint64_t replica_capacity; /* max live replicas over all workers; 0 = min(W*K, 2^24) */
+  const float* init_values;  /* K*D floats (host or device), copied at create; NULL = zeros */
+  void* stream;              /* cudaStream_t to run on; NULL = a stream owned by the library */
+} adapm_config;
+
+/* Create a manager: main store = init_values, every clock 0, no intents, no
+ * replicas.  Memory: K*D*4 (main) + W*K*6 (slot map, refcounts) + K*4
+ * (holder masks) + K*4 (scratch) + capacity*(2*D*4 + 12) bytes of device
+ * memory.  Returns ADAPM_ENOMEM if it does not fit. */
+adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out);
+
+/* Wait for outstanding work and free everything the context owns. */
+adapm_status adapm_destroy(adapm_ctx* ctx);
+
+/* Intent(keys, clock_start, clock_end) of `worker` (Sec. 3): the worker will
+ * access `keys` while clock_start <= C^worker < clock_end.  Keys are a set:
+ * repeats count once.  The optional intent type of the paper is not needed:
+ * all types are treated alike (Sec. 4.1).  An empty window (clock_end <=
+ * clock_start) or an expired one (clock_end <= C^worker) is a no-op.  A
+ * window that contains the current clock is active at once: missing
+ * replicas are created before the call's work ends.  Otherwise the keys are
+ * sorted, de-duplicated and stored until the worker's clock reaches
+ * clock_start.  Overlapping intents are reference-counted per (worker, key). */
+adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                          int64_t clock_start, int64_t clock_end);
+
+/* advanceClock() of `worker` (Sec. 3): C^worker += 1.  Replicas whose last
+ * active intent expired are destroyed (their updates merged into main), then
+ * replicas for keys whose first intent became active are created (value
+ * copied from main).  A key that stays active keeps its replica untouched. */
+adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker);
+
+/* Read n rows: out[i] = worker's replica of keys[i] if it holds one, else the
+ * main copy (Sec. 5.1: reads without replica are current).  Keys may repeat.
+ * out: n*D floats, row i for keys[i]. */
+adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                        float* out);
+
+/* Write n delta rows: the rows of each distinct key are summed and the sum is
+ * added to the worker's replica (its value and its pending-update
+ * accumulator) or, without a replica, to the main copy (Sec. 4, App. B.1.2).
+ * deltas: n*D floats, row i for keys[i].  Summation: rows in order of
+ * appearance within fixed chunks of the key-sorted batch, chunk sums in
+ * chunk order; deterministic for a given input. */
+adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                        const float* deltas);
+
+/* Replica synchronisation (App. B.1.2): for every key with replicas,
+ * main += the pending updates of all holders (ascending worker order), then
+ * every holder's replica := main and its pending updates := 0. */
+adapm_status adapm_sync(adapm_ctx* ctx);
+
+/* Block until the stream is idle; return and clear the first sticky device
+ * error (ADAPM_ERANGE, ADAPM_ENOMEM, ADAPM_ESTATE) or ADAPM_OK. */
+adapm_status adapm_wait(adapm_ctx* ctx);
+
+/* ---- fused training steps (App. C tasks) ------------------------------ */
+/* Each reads the rows it needs from the worker's replicas or the main copy
+ * (as adapm_pull), computes the loss and gradients of every sample from those
+ * values, and pushes one delta row per row occurrence (as adapm_push).  With
+ * AdaGrad the value row is [theta | a] (D = 2*dim) and a delta row is
+ * [-lr*g/sqrt(a+g*g+eps) | g*g]; without, D = dim and the delta is -lr*g.
+ * loss_out (host or device double, may be NULL) receives the batch loss sum,
+ * valid after adapm_wait(). */
+
+/* Matrix factorisation, loss 1/2 (v - u.w)^2 per cell (App. C "Matrix
+ * factorization"): row_keys[i], col_keys[i], vals[i] for i < n. */
+adapm_status adapm_mf_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* row_keys,
+                           const uint32_t* col_keys, const float* vals, uint64_t n,
+                           uint32_t dim, int adagrad, float lr, float eps, double* loss_out);
+
+/* ComplEx knowledge-graph embeddings with logistic loss (App. C "Knowledge
+ * graph embeddings"): rows [re(dim/2) | im(dim/2)] (+ AdaGrad), score
+ * Re(sum h r conj(t)); per triple i: heads[i], rels[i], tails[i] positive and
+ * neg_tails[i*n_neg + j] negative (label -1).  AdaGrad always (D = 2*dim). */
+adapm_status adapm_complex_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* heads,
+                                const uint32_t* rels, const uint32_t* tails,
+                                const uint32_t* neg_tails, uint64_t n, uint32_t n_neg,
+                                uint32_t dim, float lr, float eps, double* loss_out);
+
+/* Skip-gram with negative sampling, plain SGD (App. C "Word vectors"): input
+ * vector of token c is key c, output vector of token o is key vocab + o.
+ * centres[i]; contexts[i*n_ctx + j] (0xFFFFFFFF = no context in that slot);
+ * negatives[(i*n_ctx + j)*n_neg + q].  D = dim. */
+adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* centres,
+                             const uint32_t* contexts, const uint32_t* negatives, uint64_t n,
+                             uint32_t n_ctx, uint32_t n_neg, uint32_t vocab, uint32_t dim,
+                             float lr, double* loss_out);
+
+/* ---- inspection (synchronising; for tests and tools) ------------------ */
+adapm_status adapm_clock(adapm_ctx* ctx, uint32_t worker, int64_t* out);
+
+/* Keys of the worker's replicas in ascending order: the logical slot map
+ * (slot of key k = rank of k in this list).  Writes min(cap, count) keys to
+ * out (host or device) and the count to *n (host). */
+adapm_status adapm_replica_keys(adapm_ctx* ctx, uint32_t worker, uint32_t* out, uint64_t cap,
+                                uint64_t* n);
+
+/* For each key: has[i] = 1 if the worker holds a replica, and its value row
+ * and pending-update row (zeros when it holds none). */
+adapm_status adapm_replica_rows(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                                float* val_out, float* acc_out, uint8_t* has_out);
+
+/* Number of the worker's active intents containing each key (uint32 out). */
+adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                             uint32_t* out);
+
+/* Rows of the main copy. */
+adapm_status adapm_read_main(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, float* out);
+
+typedef struct {
+  uint64_t live_replicas;    /* replicas that exist now, all workers */
+  uint64_t high_water;       /* replica slots ever in use */
+  uint64_t capacity;
+  uint64_t created, destroyed;
+  uint64_t last_push_unique; /* distinct keys of the last push */
+} adapm_stats;
+
+adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);
+
+/* Per-operation device time: when enabled, every call records CUDA events
+ * around its work on the library stream.  Operations: 0 intent, 1 advance,
+ * 2 pull, 3 push, 4 sync, 5 training-step compute (without its push),
+ * 6 push gather-scatter kernel alone, 7 pull gather kernel alone.
+ * adapm_profile_read synchronises and returns the summed milliseconds and
+ * call counts since the last read (arrays of ADAPM_NUM_OPS). */
+#define ADAPM_NUM_OPS 8
+adapm_status adapm_profile_enable(adapm_ctx* ctx, int enable);
+adapm_status adapm_profile_read(adapm_ctx* ctx, double* ms_out, uint64_t* calls_out);
+
+/* Message for the last error returned on this context ("" if none). */
+const char* adapm_last_error(adapm_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ADAPM_H */

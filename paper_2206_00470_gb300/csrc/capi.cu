@@ -1,0 +1,783 @@
+// extern "C" entry points of libadapm (include/adapm.h) and the host-side
+// state of a context: worker clocks and the per-clock buckets of stored
+// intent lists (Sec. 3: an intent is inactive before C_start, active in
+// [C_start, C_end), expired after).  All device work is enqueued on one
+// stream; scratch comes from a context-owned stream-ordered memory pool.
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <new>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "adapm.h"
+#include "internal.cuh"
+#include "store_launch.cuh"
+
+using namespace adapm;
+
+namespace {
+
+struct IntentList {
+  uint32_t* keys = nullptr;   // device: cap sorted unique keys, then the count word
+  uint32_t* count = nullptr;
+  uint64_t cap = 0;
+};
+
+struct WorkerState {
+  int64_t clock = 0;
+  std::map<int64_t, std::vector<int64_t>> starts;   // clock -> lists whose window opens
+  std::map<int64_t, std::vector<int64_t>> ends;     // clock -> lists whose window closes
+};
+
+}  // namespace
+
+struct adapm_ctx {
+  adapm_config cfg{};
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  int device = 0;
+  int sms = kNumSms;
+  int bits = 32;
+  cudaMemPool_t pool = nullptr;
+  Store s{};
+  DevState* dstate = nullptr;
+  std::vector<WorkerState> workers;
+  std::map<int64_t, IntentList> lists;
+  int64_t next_list = 0;
+  std::string err;
+  bool broken = false;
+  bool prof = false;
+  std::vector<std::tuple<int, cudaEvent_t, cudaEvent_t>> pending;
+  std::vector<cudaEvent_t> spare_events;
+  double prof_ms[ADAPM_NUM_OPS] = {0};
+  uint64_t prof_calls[ADAPM_NUM_OPS] = {0};
+};
+
+namespace {
+
+adapm_status fail(adapm_ctx* c, adapm_status st, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return st;
+}
+
+adapm_status cuda_fail(adapm_ctx* c, cudaError_t e, const char* where) {
+  if (c) c->broken = true;
+  return fail(c, ADAPM_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+#define CK(call)                                             \
+  do {                                                       \
+    cudaError_t e_ = (call);                                 \
+    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, #call); \
+  } while (0)
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+template <class T>
+cudaError_t pool_alloc(adapm_ctx* ctx, T** p, size_t count) {
+  if (count == 0) count = 1;
+  return cudaMallocFromPoolAsync(reinterpret_cast<void**>(p), count * sizeof(T), ctx->pool,
+                                 ctx->stream);
+}
+
+void pool_free(adapm_ctx* ctx, void* p) {
+  if (p) cudaFreeAsync(p, ctx->stream);
+}
+
+// Device view of an input array; copies host arrays in.
+template <class T>
+struct Input {
+  const T* dev = nullptr;
+  T* owned = nullptr;
+};
+
+template <class T>
+cudaError_t stage_in(adapm_ctx* ctx, const T* p, size_t count, Input<T>* in) {
+  if (count == 0 || p == nullptr) {
+    in->dev = p;
+    return cudaSuccess;
+  }
+  if (is_device_ptr(p)) {
+    in->dev = p;
+    return cudaSuccess;
+  }
+  cudaError_t e = pool_alloc(ctx, &in->owned, count);
+  if (e != cudaSuccess) return e;
+  in->dev = in->owned;
+  return cudaMemcpyAsync(in->owned, p, count * sizeof(T), cudaMemcpyHostToDevice, ctx->stream);
+}
+
+// Device buffer for an output array; copied out to host arrays at finish.
+template <class T>
+struct Output {
+  T* dev = nullptr;
+  T* host = nullptr;
+  size_t count = 0;
+};
+
+template <class T>
+cudaError_t stage_out(adapm_ctx* ctx, T* p, size_t count, Output<T>* o) {
+  o->count = count;
+  if (count == 0 || is_device_ptr(p)) {
+    o->dev = p;
+    return cudaSuccess;
+  }
+  o->host = p;
+  return pool_alloc(ctx, &o->dev, count);
+}
+
+template <class T>
+cudaError_t finish_out(adapm_ctx* ctx, Output<T>* o) {
+  if (!o->host) return cudaSuccess;
+  cudaError_t e = cudaMemcpyAsync(o->host, o->dev, o->count * sizeof(T), cudaMemcpyDeviceToHost,
+                                  ctx->stream);
+  pool_free(ctx, o->dev);
+  return e;
+}
+
+struct ProfScope {
+  adapm_ctx* ctx;
+  int op;
+  cudaEvent_t a = nullptr, b = nullptr;
+  ProfScope(adapm_ctx* c, int o) : ctx(c), op(o) {
+    if (!ctx->prof) return;
+    a = take();
+    b = take();
+    if (a) cudaEventRecord(a, ctx->stream);
+  }
+  cudaEvent_t take() {
+    if (!ctx->spare_events.empty()) {
+      cudaEvent_t e = ctx->spare_events.back();
+      ctx->spare_events.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+  }
+  ~ProfScope() {
+    if (!a || !b) return;
+    cudaEventRecord(b, ctx->stream);
+    ctx->pending.emplace_back(op, a, b);
+  }
+};
+
+adapm_status check_launch(adapm_ctx* ctx, const char* where) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(ctx, e, where);
+  return ADAPM_OK;
+}
+
+adapm_status check_ctx(adapm_ctx* ctx) {
+  if (!ctx) return ADAPM_EINVAL;
+  if (ctx->broken) return fail(ctx, ADAPM_ECUDA, "context unusable after an earlier CUDA error");
+  ctx->err.clear();
+  if (cudaSetDevice(ctx->device) != cudaSuccess) return fail(ctx, ADAPM_ECUDA, "cudaSetDevice");
+  return ADAPM_OK;
+}
+
+constexpr uint64_t kMaxN = 1ull << 31;
+
+// Refcount events of one worker -> destroy, then create replicas.
+adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventList>& ev) {
+  uint64_t total = 0;
+  for (const auto& e : ev) total += e.cap;
+  if (total == 0) return ADAPM_OK;
+  uint32_t *create_list = nullptr, *evict_list = nullptr;
+  CK(pool_alloc(ctx, &create_list, total));
+  CK(pool_alloc(ctx, &evict_list, total));
+  CK(cudaMemsetAsync(&ctx->dstate->n_create, 0, 2 * sizeof(uint32_t), ctx->stream));
+  launch_events(ctx->s, w, ev.data(), (int)ev.size(), create_list, evict_list, ctx->sms, ctx->stream);
+  launch_evict_create(ctx->s, w, create_list, evict_list, total, ctx->sms, ctx->stream);
+  pool_free(ctx, create_list);
+  pool_free(ctx, evict_list);
+  return check_launch(ctx, "apply_events");
+}
+
+// Group, sum and apply n delta rows (device keys/rows); keys may hold kNoKey
+// when allow_nokey (rows the caller wants skipped).
+adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint64_t n,
+                         const float* drows, bool allow_nokey) {
+  if (n == 0) return ADAPM_OK;
+  uint32_t *ka = nullptr, *kb = nullptr, *va = nullptr, *vb = nullptr, *hist = nullptr;
+  CK(pool_alloc(ctx, &ka, n));
+  CK(pool_alloc(ctx, &kb, n));
+  CK(pool_alloc(ctx, &va, n));
+  CK(pool_alloc(ctx, &vb, n));
+  CK(pool_alloc(ctx, &hist, sort_hist_words(n)));
+  launch_prep_keys(dkeys, n, ctx->s.K, ka, ctx->dstate, allow_nokey, ctx->sms, ctx->stream);
+  uint32_t *sk = nullptr, *sp = nullptr;
+  radix_sort(ka, kb, va, vb, true, true, n, ctx->bits, hist, ctx->stream, &sk, &sp);
+  // chunks: enough for every SM to hold many groups, at least 16 rows each
+  uint64_t chunk = 16;
+  while (chunk < 128 && n / (chunk * 2) >= (uint64_t)ctx->sms * 128) chunk *= 2;
+  const uint64_t nchunks = (n + chunk - 1) / chunk;
+  float *ph = nullptr, *pt = nullptr;
+  CK(pool_alloc(ctx, &ph, nchunks * ctx->s.D));
+  CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
+  CK(cudaMemsetAsync(&ctx->dstate->last_unique, 0, sizeof(uint32_t), ctx->stream));
+  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w};
+  {
+    ProfScope ps(ctx, 6);
+    launch_push(ctx->s, a, ctx->sms, ctx->stream);
+  }
+  pool_free(ctx, ka);
+  pool_free(ctx, kb);
+  pool_free(ctx, va);
+  pool_free(ctx, vb);
+  pool_free(ctx, hist);
+  pool_free(ctx, ph);
+  pool_free(ctx, pt);
+  return check_launch(ctx, "push");
+}
+
+}  // namespace
+
+extern "C" {
+
+adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
+  if (!cfg || !out) return ADAPM_EINVAL;
+  *out = nullptr;
+  if (cfg->num_keys < 1 || cfg->num_keys >= 0xFFFFFFFFull || cfg->value_len == 0 ||
+      cfg->value_len % 4 != 0 || cfg->value_len > 1024 || cfg->num_workers < 1 ||
+      cfg->num_workers > (uint32_t)kMaxWorkers)
+    return ADAPM_EINVAL;
+  adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
+  if (!ctx) return ADAPM_ENOMEM;
+  ctx->cfg = *cfg;
+  const uint64_t K = cfg->num_keys, D = cfg->value_len, W = cfg->num_workers;
+  uint64_t S = cfg->replica_capacity;
+  if (S == 0) S = W * K < (1ull << 24) ? W * K : (1ull << 24);
+  if (S >= (1ull << 31)) S = (1ull << 31) - 1;
+  auto bail = [&](adapm_status st) {
+    adapm_destroy(ctx);
+    return st;
+  };
+  if (cudaGetDevice(&ctx->device) != cudaSuccess) return bail(ADAPM_ECUDA);
+  cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, ctx->device);
+  if (cfg->stream) {
+    ctx->stream = (cudaStream_t)cfg->stream;
+  } else {
+    if (cudaStreamCreateWithFlags(&ctx->stream, cudaStreamNonBlocking) != cudaSuccess)
+      return bail(ADAPM_ECUDA);
+    ctx->own_stream = true;
+  }
+  cudaMemPoolProps props{};
+  props.allocType = cudaMemAllocationTypePinned;
+  props.location.type = cudaMemLocationTypeDevice;
+  props.location.id = ctx->device;
+  if (cudaMemPoolCreate(&ctx->pool, &props) != cudaSuccess) return bail(ADAPM_ECUDA);
+  uint64_t keep = ~0ull;
+  cudaMemPoolSetAttribute(ctx->pool, cudaMemPoolAttrReleaseThreshold, &keep);
+  ctx->bits = bits_for(K);
+  Store& s = ctx->s;
+  s.K = K;
+  s.S = S;
+  s.D = (uint32_t)D;
+  s.W = (uint32_t)W;
+  auto dmalloc = [&](void** p, size_t bytes) { return cudaMalloc(p, bytes) == cudaSuccess; };
+  if (!dmalloc((void**)&s.main, K * D * 4) || !dmalloc((void**)&s.val, S * D * 4) ||
+      !dmalloc((void**)&s.acc, S * D * 4) || !dmalloc((void**)&s.map, W * K * 4) ||
+      !dmalloc((void**)&s.rc, W * K * 2) || !dmalloc((void**)&s.holders, K * 4) ||
+      !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
+      !dmalloc((void**)&s.ev_delta, K * 4) || !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
+    cudaGetLastError();
+    return bail(ADAPM_ENOMEM);
+  }
+  s.st = ctx->dstate;
+  cudaStream_t st = ctx->stream;
+  bool ok = true;
+  if (cfg->init_values) {
+    ok &= cudaMemcpyAsync(s.main, cfg->init_values, K * D * 4, cudaMemcpyDefault, st) == cudaSuccess;
+  } else {
+    ok &= cudaMemsetAsync(s.main, 0, K * D * 4, st) == cudaSuccess;
+  }
+  ok &= cudaMemsetAsync(s.map, 0xFF, W * K * 4, st) == cudaSuccess;   // -1: no replica
+  ok &= cudaMemsetAsync(s.rc, 0, W * K * 2, st) == cudaSuccess;
+  ok &= cudaMemsetAsync(s.holders, 0, K * 4, st) == cudaSuccess;
+  ok &= cudaMemsetAsync(s.ev_delta, 0, K * 4, st) == cudaSuccess;
+  DevState h{};
+  h.free_top = (int32_t)S;
+  ok &= cudaMemcpyAsync(ctx->dstate, &h, sizeof h, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  launch_init_pool(s.free_stack, S, s.slot_owner, st);
+  ok &= cudaStreamSynchronize(st) == cudaSuccess;
+  if (!ok || cudaGetLastError() != cudaSuccess) return bail(ADAPM_ECUDA);
+  ctx->workers.resize(W);
+  *out = ctx;
+  return ADAPM_OK;
+}
+
+adapm_status adapm_destroy(adapm_ctx* ctx) {
+  if (!ctx) return ADAPM_EINVAL;
+  cudaSetDevice(ctx->device);
+  if (ctx->stream) cudaStreamSynchronize(ctx->stream);
+  for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
+  Store& s = ctx->s;
+  void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
+                  s.ev_delta, ctx->dstate};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  for (auto& t : ctx->pending) {
+    cudaEventDestroy(std::get<1>(t));
+    cudaEventDestroy(std::get<2>(t));
+  }
+  for (auto e : ctx->spare_events) cudaEventDestroy(e);
+  if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
+  if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
+  cudaGetLastError();
+  delete ctx;
+  return ADAPM_OK;
+}
+
+adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                          int64_t clock_start, int64_t clock_end) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  if (n > kMaxN || (n > 0 && !keys)) return fail(ctx, ADAPM_EINVAL, "bad keys/n");
+  WorkerState& ws = ctx->workers[worker];
+  if (clock_end <= clock_start || clock_end <= ws.clock) return ADAPM_OK;   // never active
+  ProfScope ps(ctx, 0);
+  IntentList L;
+  L.cap = n;
+  CK(cudaMallocFromPoolAsync((void**)&L.keys, (n + 1) * sizeof(uint32_t), ctx->pool, ctx->stream));
+  L.count = L.keys + n;
+  if (n == 0) {
+    CK(cudaMemsetAsync(L.count, 0, sizeof(uint32_t), ctx->stream));
+  } else {
+    Input<uint32_t> in;
+    CK(stage_in(ctx, keys, n, &in));
+    uint32_t *ka = nullptr, *kb = nullptr, *hist = nullptr, *tmp = nullptr;
+    CK(pool_alloc(ctx, &ka, n));
+    CK(pool_alloc(ctx, &kb, n));
+    CK(pool_alloc(ctx, &hist, sort_hist_words(n)));
+    CK(pool_alloc(ctx, &tmp, compact_tmp_words(n)));
+    launch_prep_keys(in.dev, n, ctx->s.K, ka, ctx->dstate, false, ctx->sms, ctx->stream);
+    uint32_t *sk = nullptr, *sv = nullptr;
+    radix_sort(ka, kb, nullptr, nullptr, false, false, n, ctx->bits, hist, ctx->stream, &sk, &sv);
+    unique_sorted(sk, n, L.keys, L.count, tmp, ctx->stream);
+    pool_free(ctx, in.owned);
+    pool_free(ctx, ka);
+    pool_free(ctx, kb);
+    pool_free(ctx, hist);
+    pool_free(ctx, tmp);
+  }
+  const int64_t id = ctx->next_list++;
+  ctx->lists[id] = L;
+  if (clock_start <= ws.clock) {
+    // the window contains the current clock: active at once
+    st = apply_events(ctx, worker, {EventList{L.keys, L.count, L.cap, +1}});
+    if (st != ADAPM_OK) return st;
+  } else {
+    ws.starts[clock_start].push_back(id);
+  }
+  ws.ends[clock_end].push_back(id);
+  return check_launch(ctx, "intent");
+}
+
+adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  WorkerState& ws = ctx->workers[worker];
+  ws.clock += 1;
+  const int64_t c = ws.clock;
+  std::vector<EventList> ev;
+  std::vector<int64_t> closing;
+  auto it = ws.starts.find(c);
+  if (it != ws.starts.end()) {
+    for (int64_t id : it->second) {
+      const IntentList& L = ctx->lists[id];
+      ev.push_back(EventList{L.keys, L.count, L.cap, +1});
+    }
+    ws.starts.erase(it);
+  }
+  it = ws.ends.find(c);
+  if (it != ws.ends.end()) {
+    for (int64_t id : it->second) {
+      const IntentList& L = ctx->lists[id];
+      ev.push_back(EventList{L.keys, L.count, L.cap, -1});
+      closing.push_back(id);
+    }
+    ws.ends.erase(it);
+  }
+  if (ev.empty()) return ADAPM_OK;
+  ProfScope ps(ctx, 1);
+  st = apply_events(ctx, worker, ev);
+  for (int64_t id : closing) {
+    pool_free(ctx, ctx->lists[id].keys);
+    ctx->lists.erase(id);
+  }
+  return st;
+}
+
+adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                        float* out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  if (n > kMaxN || (n > 0 && (!keys || !out))) return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
+  if (n == 0) return ADAPM_OK;
+  ProfScope ps(ctx, 2);
+  Input<uint32_t> in;
+  CK(stage_in(ctx, keys, n, &in));
+  Output<float> o;
+  CK(stage_out(ctx, out, n * ctx->s.D, &o));
+  {
+    ProfScope pk(ctx, 7);
+    launch_pull(ctx->s, (int)worker, in.dev, n, o.dev, ctx->sms, ctx->stream);
+  }
+  CK(finish_out(ctx, &o));
+  pool_free(ctx, in.owned);
+  return check_launch(ctx, "pull");
+}
+
+adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                        const float* deltas) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  if (n > kMaxN || (n > 0 && (!keys || !deltas))) return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
+  if (n == 0) return ADAPM_OK;
+  ProfScope ps(ctx, 3);
+  Input<uint32_t> ik;
+  Input<float> id;
+  CK(stage_in(ctx, keys, n, &ik));
+  CK(stage_in(ctx, deltas, n * ctx->s.D, &id));
+  st = push_device(ctx, worker, ik.dev, n, id.dev, false);
+  pool_free(ctx, ik.owned);
+  pool_free(ctx, id.owned);
+  return st;
+}
+
+adapm_status adapm_sync(adapm_ctx* ctx) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  ProfScope ps(ctx, 4);
+  launch_sync(ctx->s, ctx->s.S, ctx->sms, ctx->stream);
+  return check_launch(ctx, "sync");
+}
+
+adapm_status adapm_wait(adapm_ctx* ctx) {
+  if (!ctx) return ADAPM_EINVAL;
+  if (ctx->broken) return fail(ctx, ADAPM_ECUDA, "context unusable after an earlier CUDA error");
+  cudaSetDevice(ctx->device);
+  CK(cudaStreamSynchronize(ctx->stream));
+  uint32_t errors = 0;
+  CK(cudaMemcpy(&errors, &ctx->dstate->errors, sizeof errors, cudaMemcpyDeviceToHost));
+  if (errors) CK(cudaMemset(&ctx->dstate->errors, 0, sizeof errors));
+  if (errors & ERR_KEY_RANGE) return fail(ctx, ADAPM_ERANGE, "a key >= num_keys was passed");
+  if (errors & ERR_NO_SLOTS) return fail(ctx, ADAPM_ENOMEM, "replica capacity exhausted");
+  if (errors & ERR_REFCOUNT) return fail(ctx, ADAPM_ESTATE, "intent refcount overflow");
+  return ADAPM_OK;
+}
+
+adapm_status adapm_mf_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* row_keys,
+                           const uint32_t* col_keys, const float* vals, uint64_t n, uint32_t dim,
+                           int adagrad, float lr, float eps, double* loss_out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  if (n > kMaxN / 2 || (n > 0 && (!row_keys || !col_keys || !vals)))
+    return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
+  if (dim == 0 || (adagrad ? 2 * dim : dim) != ctx->s.D)
+    return fail(ctx, ADAPM_EINVAL, "dim %u does not match value_len %u", dim, ctx->s.D);
+  Output<double> lo;
+  if (loss_out) CK(stage_out(ctx, loss_out, 1, &lo));
+  if (n == 0) {
+    if (loss_out) {
+      CK(cudaMemsetAsync(lo.dev, 0, sizeof(double), ctx->stream));
+      CK(finish_out(ctx, &lo));
+    }
+    return ADAPM_OK;
+  }
+  Input<uint32_t> ir, ic;
+  Input<float> iv;
+  CK(stage_in(ctx, row_keys, n, &ir));
+  CK(stage_in(ctx, col_keys, n, &ic));
+  CK(stage_in(ctx, vals, n, &iv));
+  const uint64_t m = 2 * n;
+  StepOut o{};
+  o.loss_blocks = step_loss_blocks(ctx->sms);
+  CK(pool_alloc(ctx, &o.dkeys, m));
+  CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
+  CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  {
+    ProfScope ps(ctx, 5);
+    launch_mf_step(ctx->s, worker, ir.dev, ic.dev, iv.dev, n, dim, adagrad != 0, lr, eps, o,
+                   ctx->sms, ctx->stream);
+  }
+  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
+  {
+    ProfScope ps(ctx, 3);
+    st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
+  }
+  if (loss_out) CK(finish_out(ctx, &lo));
+  pool_free(ctx, ir.owned);
+  pool_free(ctx, ic.owned);
+  pool_free(ctx, iv.owned);
+  pool_free(ctx, o.dkeys);
+  pool_free(ctx, o.drows);
+  pool_free(ctx, o.loss_part);
+  if (st != ADAPM_OK) return st;
+  return check_launch(ctx, "mf_step");
+}
+
+adapm_status adapm_complex_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* heads,
+                                const uint32_t* rels, const uint32_t* tails,
+                                const uint32_t* neg_tails, uint64_t n, uint32_t n_neg,
+                                uint32_t dim, float lr, float eps, double* loss_out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  if (n > kMaxN / (3 + (uint64_t)n_neg) ||
+      (n > 0 && (!heads || !rels || !tails || (n_neg > 0 && !neg_tails))))
+    return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
+  if (dim == 0 || dim % 2 != 0 || 2 * dim != ctx->s.D)
+    return fail(ctx, ADAPM_EINVAL, "dim %u: need even dim with value_len = 2*dim", dim);
+  Output<double> lo;
+  if (loss_out) CK(stage_out(ctx, loss_out, 1, &lo));
+  if (n == 0) {
+    if (loss_out) {
+      CK(cudaMemsetAsync(lo.dev, 0, sizeof(double), ctx->stream));
+      CK(finish_out(ctx, &lo));
+    }
+    return ADAPM_OK;
+  }
+  Input<uint32_t> ih, ir, it, ineg;
+  CK(stage_in(ctx, heads, n, &ih));
+  CK(stage_in(ctx, rels, n, &ir));
+  CK(stage_in(ctx, tails, n, &it));
+  CK(stage_in(ctx, neg_tails, n * n_neg, &ineg));
+  const uint64_t m = n * (3 + (uint64_t)n_neg);
+  StepOut o{};
+  o.loss_blocks = step_loss_blocks(ctx->sms);
+  CK(pool_alloc(ctx, &o.dkeys, m));
+  CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
+  CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  {
+    ProfScope ps(ctx, 5);
+    launch_complex_step(ctx->s, worker, ih.dev, ir.dev, it.dev, ineg.dev, n, n_neg, dim, lr, eps,
+                        o, ctx->sms, ctx->stream);
+  }
+  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
+  {
+    ProfScope ps(ctx, 3);
+    st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
+  }
+  if (loss_out) CK(finish_out(ctx, &lo));
+  for (void* p : {(void*)ih.owned, (void*)ir.owned, (void*)it.owned, (void*)ineg.owned,
+                  (void*)o.dkeys, (void*)o.drows, (void*)o.loss_part})
+    pool_free(ctx, p);
+  if (st != ADAPM_OK) return st;
+  return check_launch(ctx, "complex_step");
+}
+
+adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* centres,
+                             const uint32_t* contexts, const uint32_t* negatives, uint64_t n,
+                             uint32_t n_ctx, uint32_t n_neg, uint32_t vocab, uint32_t dim,
+                             float lr, double* loss_out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  const uint64_t per = 1 + (uint64_t)n_ctx * (1 + (uint64_t)n_neg);
+  if (n > kMaxN / per || (n > 0 && (!centres || (n_ctx > 0 && !contexts) ||
+                                    (n_ctx > 0 && n_neg > 0 && !negatives))))
+    return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
+  if (dim != ctx->s.D) return fail(ctx, ADAPM_EINVAL, "dim %u != value_len %u", dim, ctx->s.D);
+  if (2ull * vocab > ctx->s.K) return fail(ctx, ADAPM_EINVAL, "2*vocab exceeds num_keys");
+  Output<double> lo;
+  if (loss_out) CK(stage_out(ctx, loss_out, 1, &lo));
+  if (n == 0) {
+    if (loss_out) {
+      CK(cudaMemsetAsync(lo.dev, 0, sizeof(double), ctx->stream));
+      CK(finish_out(ctx, &lo));
+    }
+    return ADAPM_OK;
+  }
+  Input<uint32_t> ic, ix, ineg;
+  CK(stage_in(ctx, centres, n, &ic));
+  CK(stage_in(ctx, contexts, n * n_ctx, &ix));
+  CK(stage_in(ctx, negatives, n * n_ctx * n_neg, &ineg));
+  const uint64_t m = n * per;
+  StepOut o{};
+  o.loss_blocks = step_loss_blocks(ctx->sms);
+  CK(pool_alloc(ctx, &o.dkeys, m));
+  CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
+  CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  {
+    ProfScope ps(ctx, 5);
+    launch_sgns_step(ctx->s, worker, ic.dev, ix.dev, ineg.dev, n, n_ctx, n_neg, vocab, dim, lr, o,
+                     ctx->sms, ctx->stream);
+  }
+  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
+  {
+    ProfScope ps(ctx, 3);
+    st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
+  }
+  if (loss_out) CK(finish_out(ctx, &lo));
+  for (void* p : {(void*)ic.owned, (void*)ix.owned, (void*)ineg.owned, (void*)o.dkeys,
+                  (void*)o.drows, (void*)o.loss_part})
+    pool_free(ctx, p);
+  if (st != ADAPM_OK) return st;
+  return check_launch(ctx, "sgns_step");
+}
+
+adapm_status adapm_clock(adapm_ctx* ctx, uint32_t worker, int64_t* out) {
+  if (!ctx || !out) return ADAPM_EINVAL;
+  if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
+  *out = ctx->workers[worker].clock;
+  return ADAPM_OK;
+}
+
+adapm_status adapm_replica_keys(adapm_ctx* ctx, uint32_t worker, uint32_t* out, uint64_t cap,
+                                uint64_t* n) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W || !n || (cap > 0 && !out)) return fail(ctx, ADAPM_EINVAL, "bad arguments");
+  uint32_t *buf = nullptr, *tmp = nullptr, *cnt = nullptr;
+  CK(pool_alloc(ctx, &buf, ctx->s.K));
+  CK(pool_alloc(ctx, &tmp, compact_tmp_words(ctx->s.K)));
+  CK(pool_alloc(ctx, &cnt, 1));
+  compact_replica_keys(ctx->s.map + (uint64_t)worker * ctx->s.K, ctx->s.K, buf, cnt, tmp, ctx->stream);
+  uint32_t hcnt = 0;
+  CK(cudaMemcpyAsync(&hcnt, cnt, sizeof hcnt, cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  *n = hcnt;
+  const uint64_t m = hcnt < cap ? hcnt : cap;
+  if (m > 0) CK(cudaMemcpyAsync(out, buf, m * 4, cudaMemcpyDefault, ctx->stream));
+  pool_free(ctx, buf);
+  pool_free(ctx, tmp);
+  pool_free(ctx, cnt);
+  CK(cudaStreamSynchronize(ctx->stream));
+  return check_launch(ctx, "replica_keys");
+}
+
+adapm_status adapm_replica_rows(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                                float* val_out, float* acc_out, uint8_t* has_out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W || n > kMaxN || (n > 0 && (!keys || !val_out || !acc_out || !has_out)))
+    return fail(ctx, ADAPM_EINVAL, "bad arguments");
+  if (n == 0) return ADAPM_OK;
+  Input<uint32_t> in;
+  CK(stage_in(ctx, keys, n, &in));
+  Output<float> ov, oa;
+  Output<uint8_t> oh;
+  CK(stage_out(ctx, val_out, n * ctx->s.D, &ov));
+  CK(stage_out(ctx, acc_out, n * ctx->s.D, &oa));
+  CK(stage_out(ctx, has_out, n, &oh));
+  launch_replica_rows(ctx->s, worker, in.dev, n, ov.dev, oa.dev, oh.dev, ctx->stream);
+  CK(finish_out(ctx, &ov));
+  CK(finish_out(ctx, &oa));
+  CK(finish_out(ctx, &oh));
+  pool_free(ctx, in.owned);
+  CK(cudaStreamSynchronize(ctx->stream));
+  return check_launch(ctx, "replica_rows");
+}
+
+adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                             uint32_t* out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (worker >= ctx->s.W || n > kMaxN || (n > 0 && (!keys || !out)))
+    return fail(ctx, ADAPM_EINVAL, "bad arguments");
+  if (n == 0) return ADAPM_OK;
+  Input<uint32_t> in;
+  CK(stage_in(ctx, keys, n, &in));
+  Output<uint32_t> o;
+  CK(stage_out(ctx, out, n, &o));
+  launch_refcounts(ctx->s, worker, in.dev, n, o.dev, ctx->stream);
+  CK(finish_out(ctx, &o));
+  pool_free(ctx, in.owned);
+  CK(cudaStreamSynchronize(ctx->stream));
+  return check_launch(ctx, "refcounts");
+}
+
+adapm_status adapm_read_main(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, float* out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (n > kMaxN || (n > 0 && (!keys || !out))) return fail(ctx, ADAPM_EINVAL, "bad arguments");
+  if (n == 0) return ADAPM_OK;
+  Input<uint32_t> in;
+  CK(stage_in(ctx, keys, n, &in));
+  Output<float> o;
+  CK(stage_out(ctx, out, n * ctx->s.D, &o));
+  launch_pull(ctx->s, -1, in.dev, n, o.dev, ctx->sms, ctx->stream);
+  CK(finish_out(ctx, &o));
+  pool_free(ctx, in.owned);
+  CK(cudaStreamSynchronize(ctx->stream));
+  return check_launch(ctx, "read_main");
+}
+
+adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (!out) return fail(ctx, ADAPM_EINVAL, "null output");
+  DevState h{};
+  CK(cudaMemcpyAsync(&h, ctx->dstate, sizeof h, cudaMemcpyDeviceToHost, ctx->stream));
+  CK(cudaStreamSynchronize(ctx->stream));
+  out->live_replicas = (uint64_t)(h.live > 0 ? h.live : 0);
+  out->high_water = (uint64_t)h.high_water;
+  out->capacity = ctx->s.S;
+  out->created = h.created;
+  out->destroyed = h.destroyed;
+  out->last_push_unique = h.last_unique;
+  return ADAPM_OK;
+}
+
+adapm_status adapm_profile_enable(adapm_ctx* ctx, int enable) {
+  if (!ctx) return ADAPM_EINVAL;
+  ctx->prof = enable != 0;
+  return ADAPM_OK;
+}
+
+adapm_status adapm_profile_read(adapm_ctx* ctx, double* ms_out, uint64_t* calls_out) {
+  if (!ctx) return ADAPM_EINVAL;
+  cudaSetDevice(ctx->device);
+  CK(cudaStreamSynchronize(ctx->stream));
+  for (auto& t : ctx->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, std::get<1>(t), std::get<2>(t)) == cudaSuccess) {
+      ctx->prof_ms[std::get<0>(t)] += ms;
+      ctx->prof_calls[std::get<0>(t)] += 1;
+    }
+    ctx->spare_events.push_back(std::get<1>(t));
+    ctx->spare_events.push_back(std::get<2>(t));
+  }
+  ctx->pending.clear();
+  cudaGetLastError();
+  for (int i = 0; i < ADAPM_NUM_OPS; ++i) {
+    if (ms_out) ms_out[i] = ctx->prof_ms[i];
+    if (calls_out) calls_out[i] = ctx->prof_calls[i];
+    ctx->prof_ms[i] = 0;
+    ctx->prof_calls[i] = 0;
+  }
+  return ADAPM_OK;
+}
+
+const char* adapm_last_error(adapm_ctx* ctx) {
+  if (!ctx) return "null context";
+  return ctx->err.c_str();
+}
+
+}  // extern "C"

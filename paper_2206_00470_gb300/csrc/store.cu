@@ -1,0 +1,692 @@
+// Kernels of the parameter manager's hot path.
+//
+// Rows are moved as float4 (128-bit) by "row groups" of G lanes, each lane
+// owning columns lane, lane+G, ..., lane+(C-1)G of a row (D4 = D/4 <= G*C).
+// Kernels are persistent grids (a multiple of the SM count) with several
+// independent rows in flight per group (R-way unrolled address chains:
+// key -> slot -> row), which is what an HBM-bound gather needs.
+//
+//   pull        out[i] = replica of keys[i] at worker w, else main       (Sec. 5.1)
+//   push        sorted (key, position) pairs are split into fixed chunks;
+//               each group sums the delta rows of every key segment of its
+//               chunk in position order and adds the sum to the worker's
+//               replica (value and pending updates) or to main (Sec. 4,
+//               App. B.1.2); segments cut by a chunk boundary leave partial
+//               sums that one owner combines in chunk order (fix-up)
+//   events      net refcount change per key of one advance, transitions
+//               0 -> >0 (create) and >0 -> 0 (evict)                    (Sec. 3)
+//   evict       main += pending updates; free the slot                 (Sec. 4.1)
+//   create      val = main, pending = 0; take a slot                   (Sec. 4.1)
+//   sync        main += sum of all holders' pending updates (ascending
+//               worker), holders := main, pending := 0                 (App. B.1.2)
+#include "internal.cuh"
+#include "store_launch.cuh"
+
+namespace adapm {
+
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ float4 f4add(float4 a, float4 b) {
+  return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float4 f4zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
+
+template <int G>
+__device__ __forceinline__ uint64_t group_id() {
+  return ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
+}
+template <int G>
+__device__ __forceinline__ uint64_t group_count() {
+  return ((uint64_t)gridDim.x * blockDim.x) / G;
+}
+
+// ---------------------------------------------------------------------------
+// key preparation: copy, range check, sentinel for bad keys
+// ---------------------------------------------------------------------------
+__global__ void prep_keys_kernel(const uint32_t* __restrict__ in, uint64_t n, uint64_t K,
+                                 uint32_t* __restrict__ out, DevState* st, int allow_nokey) {
+  bool bad = false;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (uint64_t)gridDim.x * blockDim.x) {
+    uint32_t k = in[i];
+    if (k >= K) {
+      if (!(allow_nokey && k == kNoKey)) bad = true;
+      k = kNoKey;
+    }
+    out[i] = k;
+  }
+  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(st, ERR_KEY_RANGE);
+}
+
+// ---------------------------------------------------------------------------
+// pull (and main-only gather for inspection when w < 0)
+// ---------------------------------------------------------------------------
+template <int G, int C, int R>
+__global__ void __launch_bounds__(kThreads)
+pull_kernel(Store s, int w, const uint32_t* __restrict__ keys, uint64_t n, float* __restrict__ out) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const uint32_t D4 = s.D >> 2;
+  const float4* main4 = reinterpret_cast<const float4*>(s.main);
+  const float4* val4 = reinterpret_cast<const float4*>(s.val);
+  float4* out4 = reinterpret_cast<float4*>(out);
+  const int32_t* mapw = w >= 0 ? s.map + (uint64_t)w * s.K : nullptr;
+  bool bad = false;
+  for (uint64_t base = g * R; base < n; base += ng * R) {
+    uint32_t k[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) k[r] = base + r < n ? __ldg(keys + base + r) : kNoKey;
+    int32_t sl[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) sl[r] = (mapw != nullptr && k[r] < s.K) ? __ldg(mapw + k[r]) : -1;
+    const float4* src[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      src[r] = nullptr;
+      if (k[r] < s.K) src[r] = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
+      else if (base + r < n) bad = true;
+    }
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4) {
+        float4 v[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) v[r] = src[r] != nullptr ? __ldg(src[r] + col) : f4zero();
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+          if (base + r < n) __stcs(out4 + (base + r) * D4 + col, v[r]);
+      }
+    }
+  }
+  if (bad && lane == 0) set_error(s.st, ERR_KEY_RANGE);
+}
+
+// ---------------------------------------------------------------------------
+// push: chunked segmented reduction over key-sorted (key, position) pairs
+// ---------------------------------------------------------------------------
+template <int C>
+__device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, uint32_t k,
+                                          const float4 (&sum)[C], int lane, int G) {
+  const uint32_t D4 = s.D >> 2;
+  const int32_t sl = mapw[k];
+  float4* val4 = reinterpret_cast<float4*>(s.val);
+  float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  float4* main4 = reinterpret_cast<float4*>(s.main);
+  float4* t1 = sl >= 0 ? val4 + (uint64_t)sl * D4 : main4 + (uint64_t)k * D4;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const uint32_t col = lane + c * G;
+    if (col < D4) t1[col] = f4add(t1[col], sum[c]);
+  }
+  if (sl >= 0) {
+    float4* t2 = acc4 + (uint64_t)sl * D4;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4) t2[col] = f4add(t2[col], sum[c]);
+    }
+  }
+}
+
+template <int G, int C, int R>
+__global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs a) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const uint32_t D4 = s.D >> 2;
+  const float4* d4 = reinterpret_cast<const float4*>(a.deltas);
+  float4* val4 = reinterpret_cast<float4*>(s.val);
+  float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  float4* main4 = reinterpret_cast<float4*>(s.main);
+  float4* ph4 = reinterpret_cast<float4*>(a.part_head);
+  float4* pt4 = reinterpret_cast<float4*>(a.part_tail);
+  const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
+  uint32_t heads = 0;
+  for (uint64_t j = g; j < a.nchunks; j += ng) {
+    const uint64_t p0 = j * a.chunk;
+    const uint64_t p1 = p0 + a.chunk < a.n ? p0 + a.chunk : a.n;
+    const bool has_prev = p0 > 0;
+    const uint32_t prev_key = has_prev ? a.skeys[p0 - 1] : 0u;
+    const bool has_after = p1 < a.n;
+    const uint32_t after_key = has_after ? a.skeys[p1] : 0u;
+    uint32_t cur = 0;
+    bool cur_valid = false, cur_started = false;
+    float4 run[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) run[c] = f4zero();
+    for (uint64_t p = p0; p < p1; p += R) {
+      uint32_t k[R], src[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        const bool v = p + r < p1;
+        k[r] = v ? a.skeys[p + r] : kNoKey;
+        src[r] = v ? a.spos[p + r] : 0u;
+      }
+      const bool q_in = p + R < p1;
+      const uint32_t knext = q_in ? a.skeys[p + R] : after_key;
+      const bool knext_valid = q_in || has_after;
+      float4 d[R][C];
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          d[r][c] = (p + r < p1 && k[r] != kNoKey && col < D4)
+                        ? __ldg(d4 + (uint64_t)src[r] * D4 + col) : f4zero();
+        }
+      }
+      uint32_t fl[R];   // bit0 piece ends here, bit1 piece started in chunk, bit2 segment ends here
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        fl[r] = 0;
+        if (p + r < p1) {
+          if (!cur_valid || k[r] != cur) {
+            cur = k[r];
+            cur_valid = true;
+            cur_started = (p + r > p0) || !has_prev || prev_key != k[r];
+            if (cur_started && k[r] != kNoKey) ++heads;
+#pragma unroll
+            for (int c = 0; c < C; ++c) run[c] = f4zero();
+          }
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            run[c] = f4add(run[c], d[r][c]);
+            d[r][c] = run[c];
+          }
+          bool kn_valid;
+          uint32_t kn;
+          if (r + 1 < R && p + r + 1 < p1) {
+            kn = k[r + 1];
+            kn_valid = true;
+          } else {
+            kn = knext;
+            kn_valid = knext_valid;
+          }
+          const bool seg_end = !kn_valid || kn != k[r];
+          const bool last = (p + r + 1 == p1);
+          fl[r] = ((seg_end || last) ? 1u : 0u) | (cur_started ? 2u : 0u) | (seg_end ? 4u : 0u);
+          if (k[r] == kNoKey) fl[r] = 0;
+        }
+      }
+      // whole segments inside the chunk: add straight into their target
+      int32_t sl[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) sl[r] = fl[r] == 7u ? mapw[k[r]] : -2;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) {
+          float4 t[R];
+#pragma unroll
+          for (int r = 0; r < R; ++r)
+            if (sl[r] != -2)
+              t[r] = sl[r] >= 0 ? val4[(uint64_t)sl[r] * D4 + col] : main4[(uint64_t)k[r] * D4 + col];
+#pragma unroll
+          for (int r = 0; r < R; ++r) {
+            if (sl[r] != -2) {
+              float4* dst = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
+              dst[col] = f4add(t[r], d[r][c]);
+            }
+          }
+#pragma unroll
+          for (int r = 0; r < R; ++r)
+            if (sl[r] >= 0) t[r] = acc4[(uint64_t)sl[r] * D4 + col];
+#pragma unroll
+          for (int r = 0; r < R; ++r)
+            if (sl[r] >= 0) acc4[(uint64_t)sl[r] * D4 + col] = f4add(t[r], d[r][c]);
+        }
+      }
+      // pieces of segments cut by a chunk boundary: partial sums
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if ((fl[r] & 1u) && fl[r] != 7u) {
+          float4* dst = (fl[r] & 2u) ? pt4 : ph4;
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            if (col < D4) dst[j * D4 + col] = d[r][c];
+          }
+        }
+      }
+    }
+  }
+  if (lane == 0 && heads) atomicAdd(&s.st->last_unique, heads);
+}
+
+// A segment that starts in chunk j and continues past it is owned by j:
+// tail piece of j + head pieces of j+1 .. m_end, in chunk order.
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs a) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const uint32_t D4 = s.D >> 2;
+  const float4* ph4 = reinterpret_cast<const float4*>(a.part_head);
+  const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
+  const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
+  for (uint64_t j = g; j < a.nchunks; j += ng) {
+    const uint64_t p0 = j * a.chunk;
+    const uint64_t p1 = p0 + a.chunk;
+    if (p1 >= a.n) continue;
+    const uint32_t kl = a.skeys[p1 - 1];
+    if (kl == kNoKey || a.skeys[p1] != kl) continue;
+    if (p0 > 0 && a.skeys[p0 - 1] == kl) continue;           // started in an earlier chunk
+    // last chunk m whose first position still holds kl (monotone predicate)
+    uint64_t lo = j + 1, hi = a.nchunks - 1;
+    while (lo < hi) {
+      const uint64_t mid = (lo + hi + 1) / 2;
+      if (a.skeys[mid * a.chunk] == kl) lo = mid; else hi = mid - 1;
+    }
+    const uint64_t m_end = lo;
+    float4 tot[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
+    }
+    constexpr int U = 8 / C > 0 ? 8 / C : 1;
+    for (uint64_t m = j + 1; m <= m_end; m += U) {
+      float4 t[U][C];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          t[u][c] = (m + u <= m_end && col < D4) ? ph4[(m + u) * D4 + col] : f4zero();
+        }
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (m + u <= m_end)
+#pragma unroll
+          for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+    }
+    apply_sum<C>(s, mapw, kl, tot, lane, G);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// intent events -> refcounts -> create / evict lists
+// ---------------------------------------------------------------------------
+__global__ void events_add_kernel(const uint32_t* __restrict__ keys, const uint32_t* __restrict__ count,
+                                  int sign, int32_t* __restrict__ ev_delta) {
+  const uint32_t n = *count;
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+    atomicAdd(ev_delta + keys[i], sign);
+}
+
+__device__ __forceinline__ uint32_t lanemask_lt_() {
+  uint32_t m;
+  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+  return m;
+}
+
+// warp-aggregated append to a device list
+__device__ __forceinline__ void warp_append(bool want, uint32_t value, uint32_t* counter, uint32_t* list) {
+  const uint32_t m = __ballot_sync(0xFFFFFFFFu, want);
+  if (m == 0) return;
+  const int leader = __ffs(m) - 1;
+  uint32_t base = 0;
+  if ((int)(threadIdx.x & 31) == leader) base = atomicAdd(counter, (uint32_t)__popc(m));
+  base = __shfl_sync(0xFFFFFFFFu, base, leader);
+  if (want) list[base + __popc(m & lanemask_lt_())] = value;
+}
+
+__global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys,
+                                    const uint32_t* __restrict__ count, uint32_t* create_list,
+                                    uint32_t* evict_list) {
+  const uint32_t n = *count;
+  uint16_t* rcw = s.rc + (uint64_t)w * s.K;
+  const uint32_t stride = gridDim.x * blockDim.x;
+  for (uint32_t b = blockIdx.x * blockDim.x; b < n; b += stride) {   // warp-uniform trip count
+    const uint32_t i = b + threadIdx.x;
+    bool create = false, evict = false;
+    uint32_t k = 0;
+    if (i < n) {
+      k = keys[i];
+      const int32_t d = atomicExch(s.ev_delta + k, 0);
+      if (d != 0) {
+        const int32_t old = rcw[k];
+        int32_t nw = old + d;
+        if (nw < 0 || nw > 65535) {
+          set_error(s.st, ERR_REFCOUNT);
+          nw = nw < 0 ? 0 : 65535;
+        }
+        rcw[k] = (uint16_t)nw;
+        create = old == 0 && nw > 0;
+        evict = old > 0 && nw == 0;
+      }
+    }
+    warp_append(create, k, &s.st->n_create, create_list);
+    warp_append(evict, k, &s.st->n_evict, evict_list);
+  }
+}
+
+// evict: main[k] += acc[slot]; release slot
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads) evict_kernel(Store s, uint32_t w, const uint32_t* __restrict__ list) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint32_t D4 = s.D >> 2;
+  const uint32_t n = s.st->n_evict;
+  int32_t* mapw = s.map + (uint64_t)w * s.K;
+  float4* main4 = reinterpret_cast<float4*>(s.main);
+  const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
+  constexpr int GPW = 32 / G;   // groups per warp
+  const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint64_t nwarps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  const int gi = (threadIdx.x & 31) / G;
+  for (uint64_t b = warp * GPW; b < n; b += nwarps * GPW) {
+    const uint64_t i = b + gi;
+    int32_t sl = -1;
+    uint32_t k = 0;
+    if (i < n) {
+      k = list[i];
+      sl = mapw[k];
+    }
+    if (sl >= 0) {
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) main4[(uint64_t)k * D4 + col] = f4add(main4[(uint64_t)k * D4 + col], acc4[(uint64_t)sl * D4 + col]);
+      }
+    }
+    const bool rel = sl >= 0 && lane == 0;
+    const uint32_t m = __ballot_sync(0xFFFFFFFFu, rel);
+    if (m) {
+      const int leader = __ffs(m) - 1;
+      int32_t base = 0;
+      if ((int)(threadIdx.x & 31) == leader) {
+        base = atomicAdd(&s.st->free_top, (int32_t)__popc(m));
+        atomicSub(&s.st->live, (int32_t)__popc(m));
+        atomicAdd(&s.st->destroyed, (unsigned long long)__popc(m));
+      }
+      base = __shfl_sync(0xFFFFFFFFu, base, leader);
+      if (rel) {
+        mapw[k] = -1;
+        atomicAnd(s.holders + k, ~(1u << w));
+        s.slot_owner[sl] = kEmptySlot;
+        s.free_stack[base + __popc(m & lanemask_lt_())] = sl;
+      }
+    }
+  }
+}
+
+__global__ void alloc_kernel(DevState* st) {
+  const uint32_t n = st->n_create;
+  if ((int64_t)n > (int64_t)st->free_top) {
+    st->errors |= ERR_NO_SLOTS;
+    st->n_create_ok = 0;
+    st->alloc_base = st->free_top;
+    return;
+  }
+  st->alloc_base = st->free_top - (int32_t)n;
+  st->free_top = st->alloc_base;
+  st->n_create_ok = n;
+  st->live += (int32_t)n;
+  st->created += n;
+}
+
+// create: val = main[k], acc = 0, take a slot from the stack
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, const uint32_t* __restrict__ list) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint32_t D4 = s.D >> 2;
+  const uint32_t n = s.st->n_create_ok;
+  const int32_t base = s.st->alloc_base;
+  int32_t* mapw = s.map + (uint64_t)w * s.K;
+  const float4* main4 = reinterpret_cast<const float4*>(s.main);
+  float4* val4 = reinterpret_cast<float4*>(s.val);
+  float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  int32_t hw = 0;
+  for (uint64_t i = g; i < n; i += ng) {
+    const uint32_t k = list[i];
+    // slots popped from the top of the stack: lowest free slots come first
+    const int32_t sl = s.free_stack[base + (int32_t)(n - 1 - i)];
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4) {
+        val4[(uint64_t)sl * D4 + col] = main4[(uint64_t)k * D4 + col];
+        acc4[(uint64_t)sl * D4 + col] = f4zero();
+      }
+    }
+    if (lane == 0) {
+      mapw[k] = sl;
+      atomicOr(s.holders + k, 1u << w);
+      s.slot_owner[sl] = ((unsigned long long)w << 32) | k;
+      hw = hw > sl + 1 ? hw : sl + 1;
+    }
+  }
+  if (lane == 0 && hw > 0) atomicMax(&s.st->high_water, hw);
+}
+
+// ---------------------------------------------------------------------------
+// sync
+// ---------------------------------------------------------------------------
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
+  const int lane = threadIdx.x & (G - 1);
+  const uint32_t D4 = s.D >> 2;
+  const uint64_t hw = (uint64_t)s.st->high_water;
+  float4* main4 = reinterpret_cast<float4*>(s.main);
+  float4* val4 = reinterpret_cast<float4*>(s.val);
+  float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  for (uint64_t sl = g; sl < hw; sl += ng) {
+    const unsigned long long owner = s.slot_owner[sl];
+    if (owner == kEmptySlot) continue;
+    const uint32_t w = (uint32_t)(owner >> 32);
+    const uint32_t k = (uint32_t)owner;
+    const uint32_t mask = s.holders[k];
+    if ((uint32_t)(__ffs(mask) - 1) != w) continue;   // the lowest holder merges
+    float4 m[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
+    }
+    constexpr int Q = 8 / C > 0 ? 8 / C : 1;
+    uint32_t mm = mask;
+    while (mm) {
+      int32_t hs[Q];
+#pragma unroll
+      for (int q = 0; q < Q; ++q) {
+        hs[q] = -1;
+        if (mm) {
+          const uint32_t b = __ffs(mm) - 1;
+          mm &= mm - 1;
+          hs[q] = s.map[(uint64_t)b * s.K + k];
+        }
+      }
+      float4 t[Q][C];
+#pragma unroll
+      for (int q = 0; q < Q; ++q)
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
+        }
+#pragma unroll
+      for (int q = 0; q < Q; ++q)
+        if (hs[q] >= 0)
+#pragma unroll
+          for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
+    }
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
+    }
+    mm = mask;
+    while (mm) {
+      const uint32_t b = __ffs(mm) - 1;
+      mm &= mm - 1;
+      const int32_t h = s.map[(uint64_t)b * s.K + k];
+      if (h < 0) continue;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) {
+          val4[(uint64_t)h * D4 + col] = m[c];
+          acc4[(uint64_t)h * D4 + col] = f4zero();
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// inspection
+// ---------------------------------------------------------------------------
+__global__ void refcounts_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys, uint64_t n,
+                                 uint32_t* __restrict__ out) {
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t k = keys[i];
+    if (k < s.K) out[i] = s.rc[(uint64_t)w * s.K + k];
+    else {
+      out[i] = 0;
+      set_error(s.st, ERR_KEY_RANGE);
+    }
+  }
+}
+
+__global__ void replica_rows_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys, uint64_t n,
+                                    float* __restrict__ val_out, float* __restrict__ acc_out,
+                                    uint8_t* __restrict__ has_out) {
+  const uint32_t D = s.D;
+  for (uint64_t i = blockIdx.x; i < n; i += gridDim.x) {
+    const uint32_t k = keys[i];
+    const int32_t sl = k < s.K ? s.map[(uint64_t)w * s.K + k] : -1;
+    if (threadIdx.x == 0) {
+      has_out[i] = sl >= 0 ? 1 : 0;
+      if (k >= s.K) set_error(s.st, ERR_KEY_RANGE);
+    }
+    for (uint32_t c = threadIdx.x; c < D; c += blockDim.x) {
+      val_out[i * D + c] = sl >= 0 ? s.val[(uint64_t)sl * D + c] : 0.f;
+      acc_out[i * D + c] = sl >= 0 ? s.acc[(uint64_t)sl * D + c] : 0.f;
+    }
+  }
+}
+
+__global__ void init_pool_kernel(int32_t* free_stack, uint64_t S, unsigned long long* owner) {
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < S;
+       i += (uint64_t)gridDim.x * blockDim.x) {
+    free_stack[i] = (int32_t)(S - 1 - i);   // top of the stack holds slot 0
+    owner[i] = kEmptySlot;
+  }
+}
+
+template <typename F>
+void dispatch_gc(uint32_t D4, F&& f) {
+  if (D4 <= 4) f(std::integral_constant<int, 4>{}, std::integral_constant<int, 1>{});
+  else if (D4 <= 8) f(std::integral_constant<int, 8>{}, std::integral_constant<int, 1>{});
+  else if (D4 <= 16) f(std::integral_constant<int, 16>{}, std::integral_constant<int, 1>{});
+  else if (D4 <= 32) f(std::integral_constant<int, 32>{}, std::integral_constant<int, 1>{});
+  else if (D4 <= 64) f(std::integral_constant<int, 32>{}, std::integral_constant<int, 2>{});
+  else if (D4 <= 128) f(std::integral_constant<int, 32>{}, std::integral_constant<int, 4>{});
+  else f(std::integral_constant<int, 32>{}, std::integral_constant<int, 8>{});
+}
+
+unsigned grid_for(uint64_t groups, int G, int sms) {
+  const uint64_t per_block = kThreads / G;
+  uint64_t b = (groups + per_block - 1) / per_block;
+  const uint64_t cap = (uint64_t)sms * 8;
+  if (b > cap) b = cap;
+  if (b < 1) b = 1;
+  return (unsigned)b;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+void launch_prep_keys(const uint32_t* in, uint64_t n, uint64_t K, uint32_t* out, DevState* st,
+                      bool allow_nokey, int sms, cudaStream_t stream) {
+  if (n == 0) return;
+  uint64_t b = (n + kThreads - 1) / kThreads;
+  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+  prep_keys_kernel<<<(unsigned)b, kThreads, 0, stream>>>(in, n, K, out, st, allow_nokey ? 1 : 0);
+}
+
+void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
+                 cudaStream_t stream) {
+  if (n == 0) return;
+  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    constexpr int R = 8 / C > 0 ? 8 / C : 1;
+    pull_kernel<G, C, R><<<grid_for((n + R - 1) / R, G, sms), kThreads, 0, stream>>>(s, w, keys, n, out);
+  });
+}
+
+void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream) {
+  if (a.n == 0) return;
+  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    constexpr int R = 8 / C > 0 ? 8 / C : 1;
+    push_chunks_kernel<G, C, R><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a);
+    push_fixup_kernel<G, C><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a);
+  });
+}
+
+void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
+                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
+  for (int i = 0; i < nlists; ++i) {
+    uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
+    if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+    if (b == 0) continue;
+    events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(lists[i].keys, lists[i].count,
+                                                            lists[i].sign, s.ev_delta);
+  }
+  for (int i = 0; i < nlists; ++i) {
+    uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
+    if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+    if (b == 0) continue;
+    events_apply_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, lists[i].keys, lists[i].count,
+                                                              create_list, evict_list);
+  }
+}
+
+void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
+                         const uint32_t* evict_list, uint64_t max_events, int sms,
+                         cudaStream_t stream) {
+  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    const unsigned grid = grid_for(max_events, G, sms);
+    evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list);
+    alloc_kernel<<<1, 1, 0, stream>>>(s.st);
+    create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, create_list);
+  });
+}
+
+void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stream) {
+  if (slot_bound == 0) return;
+  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    sync_kernel<G, C><<<grid_for(slot_bound, G, sms), kThreads, 0, stream>>>(s);
+  });
+}
+
+void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, uint32_t* out,
+                      cudaStream_t stream) {
+  if (n == 0) return;
+  refcounts_kernel<<<(unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, stream>>>(
+      s, w, keys, n, out);
+}
+
+void launch_replica_rows(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, float* val,
+                         float* acc, uint8_t* has, cudaStream_t stream) {
+  if (n == 0) return;
+  replica_rows_kernel<<<(unsigned)(n < 4096 ? n : 4096), 128, 0, stream>>>(s, w, keys, n, val, acc, has);
+}
+
+void launch_init_pool(int32_t* free_stack, uint64_t S, unsigned long long* owner, cudaStream_t stream) {
+  uint64_t b = (S + 255) / 256;
+  if (b > 65535) b = 65535;
+  if (b == 0) return;
+  init_pool_kernel<<<(unsigned)b, 256, 0, stream>>>(free_stack, S, owner);
+}
+
+}  // namespace adapm

@@ -1,0 +1,73 @@
+// Host-side launchers of the store kernels (store.cu) and step kernels (steps.cu).
+#pragma once
+
+#include "internal.cuh"
+
+namespace adapm {
+
+// Arguments of the chunked push reduction.  skeys/spos: key-sorted keys and
+// their positions in `deltas` (n rows of D floats).  part_head / part_tail:
+// nchunks x D floats of scratch for segments cut by chunk boundaries.
+struct PushArgs {
+  const uint32_t* skeys;
+  const uint32_t* spos;
+  uint64_t n;
+  const float* deltas;
+  float* part_head;
+  float* part_tail;
+  uint64_t chunk;
+  uint64_t nchunks;
+  uint32_t worker;
+};
+
+// One stored intent list (sorted unique keys, device count) and the sign of
+// its refcount event: +1 when its window opens, -1 when it closes.
+struct EventList {
+  const uint32_t* keys;
+  const uint32_t* count;
+  uint64_t cap;
+  int sign;
+};
+
+void launch_prep_keys(const uint32_t* in, uint64_t n, uint64_t K, uint32_t* out, DevState* st,
+                      bool allow_nokey, int sms, cudaStream_t stream);
+void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
+                 cudaStream_t stream);
+void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream);
+void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
+                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream);
+void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
+                         const uint32_t* evict_list, uint64_t max_events, int sms,
+                         cudaStream_t stream);
+void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stream);
+void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, uint32_t* out,
+                      cudaStream_t stream);
+void launch_replica_rows(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, float* val,
+                         float* acc, uint8_t* has, cudaStream_t stream);
+void launch_init_pool(int32_t* free_stack, uint64_t S, unsigned long long* owner, cudaStream_t stream);
+
+// Fused training steps (steps.cu): read rows through the worker's slot map,
+// write one delta row per row occurrence (keys to dkeys, rows to drows) and
+// the per-block loss partials to loss_part; then the caller pushes.
+struct StepOut {
+  uint32_t* dkeys;
+  float* drows;
+  double* loss_part;     // grid-sized partial sums
+  unsigned loss_blocks;  // number of partials written
+};
+
+void launch_mf_step(const Store& s, uint32_t w, const uint32_t* rows, const uint32_t* cols,
+                    const float* vals, uint64_t n, uint32_t dim, bool adagrad, float lr, float eps,
+                    const StepOut& o, int sms, cudaStream_t stream);
+void launch_complex_step(const Store& s, uint32_t w, const uint32_t* heads, const uint32_t* rels,
+                         const uint32_t* tails, const uint32_t* negs, uint64_t n, uint32_t n_neg,
+                         uint32_t dim, float lr, float eps, const StepOut& o, int sms,
+                         cudaStream_t stream);
+void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const uint32_t* contexts,
+                      const uint32_t* negs, uint64_t n, uint32_t n_ctx, uint32_t n_neg,
+                      uint32_t vocab, uint32_t dim, float lr, const StepOut& o, int sms,
+                      cudaStream_t stream);
+unsigned step_loss_blocks(int sms);
+void launch_loss_reduce(const double* part, unsigned nparts, double* out, cudaStream_t stream);
+
+}  // namespace adapm

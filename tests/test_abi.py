@@ -1,0 +1,68 @@
+"""The C-ABI library builds, loads and exports every symbol include/adapm.h declares.
+
+No compute call is made here (no GPU needed).
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2206_00470_gb300 import adapm
+from paper_2206_00470_gb300 import build as libbuild
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "adapm.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:adapm_status|const char\*)\s+(adapm_\w+)\s*\(", text, re.M)))
+
+
+@pytest.fixture(scope="module")
+def lib_path():
+    return libbuild.build()
+
+
+def test_header_declares_the_north_star_calls():
+    names = declared_functions()
+    for n in ("adapm_create", "adapm_intent", "adapm_advance_clock", "adapm_pull", "adapm_push",
+              "adapm_sync"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib_path):
+    lib = ctypes.CDLL(lib_path)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_binding_covers_every_declared_symbol(lib_path):
+    assert sorted(adapm.EXPORTS) == declared_functions()
+    adapm.load(lib_path)
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path):
+    saved = adapm._lib
+    adapm._lib = None
+    try:
+        with pytest.raises(RuntimeError):
+            adapm.load(str(tmp_path / "missing.so"))
+    finally:
+        adapm._lib = saved
+
+
+def test_create_rejects_bad_configs_without_touching_the_gpu(lib_path):
+    lib = adapm.load(lib_path)
+    h = ctypes.c_void_p()
+    bad = [
+        adapm.Config(0, 4, 1, 0, None, None),          # no keys
+        adapm.Config(10, 6, 1, 0, None, None),         # value_len not a multiple of 4
+        adapm.Config(10, 4, 0, 0, None, None),         # no workers
+        adapm.Config(10, 4, 33, 0, None, None),        # more than 32 workers
+        adapm.Config(2 ** 32 - 1, 4, 1, 0, None, None),
+    ]
+    for cfg in bad:
+        assert lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h)) == adapm.EINVAL
+    assert lib.adapm_intent(None, 0, None, 0, 0, 1) == adapm.EINVAL
+    assert lib.adapm_wait(None) == adapm.EINVAL
