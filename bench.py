@@ -1,0 +1,611 @@
+"""Throughput of the intent-driven parameter manager on one or more GB300s.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload mf|micro|complex|sgns|tiny_mf]
+                    [--impl ours|reference]
+
+A step is one clock of the whole job: every worker slot signals the intent of
+the batch `lookahead` clocks ahead, reads and writes the rows of its current
+batch (pull + push, or one fused training step that reads through the slot
+map and pushes its delta rows), advances its clock; then one sync merges all
+replica updates (the per-clock loop of Fig. 2).  Inputs are seeded synthetic
+data resident in HBM before timing starts; the stores (9-26 GB) and per-step
+row traffic exceed the 129 MB L2, so no flush is needed between steps.
+
+Reported (one JSON line on rank 0): pulled + pushed keys/s (value), training
+samples/s, per-operation device time and algorithmic GB/s, the roofline of
+the dominant kernel against the measured HBM copy peak, the end-to-end rate
+through the C ABI with pinned host buffers (host<->device copies timed), the
+CPU oracle's rate on a bounded sample, SM clocks sampled during the timed
+region, and the number of library kernels launched in it.
+
+With --gpus N > 1 (torchrun) every rank runs an independent replica of the
+workload on its own GPU: the path has no exchange step (replicas only).
+"""
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from synth import hashgen  # noqa: E402
+from synth import workloads as wl  # noqa: E402
+
+METRIC = "pulled+pushed keys/s"
+UNIT = "keys/s"
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (timing only; the data path has no collective)
+# ---------------------------------------------------------------------------
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def init_dist(ws, backend):
+    if ws > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend)
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, ws, device):
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, ws, device):
+    if ws == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# workloads
+# ---------------------------------------------------------------------------
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+class Micro:
+    """Parameter-access microbenchmark: 100M keys x 64 fp32, Zipf keys, pull + push per worker."""
+
+    def __init__(self, args, device):
+        import dataclasses
+        self.cfg = dataclasses.replace(wl.MICRO, batch=args.batch or wl.MICRO.batch,
+                                       zipf_s=args.zipf if args.zipf is not None else wl.MICRO.zipf_s,
+                                       span=args.span or wl.MICRO.span,
+                                       num_keys=args.keys or wl.MICRO.num_keys)
+        c = self.cfg
+        self.device = device
+        self.K, self.D, self.W = c.num_keys, c.value_len, c.workers
+        self.lookahead, self.span = c.lookahead, c.span
+        self.row = self.D * 4
+        self.capacity = min(self.W * (c.span + 1) * c.batch, 80_000_000)
+        self.samples_per_step = 0
+
+    def config(self):
+        c = self.cfg
+        return {"workload": c.name, "num_keys": c.num_keys, "value_len": c.value_len,
+                "workers": c.workers, "batch_per_worker": c.batch, "zipf_s": c.zipf_s,
+                "intent_span": c.span, "lookahead": c.lookahead}
+
+    def init_store(self):
+        return hashgen.init_store_torch(self.K, self.D, self.D, self.cfg.seed, self.cfg.init_std,
+                                        self.device, chunk_rows=1 << 22)
+
+    def prepare(self, clocks):
+        c = self.cfg
+        self.keys = {}
+        for cl in range(clocks + self.lookahead + 1):
+            for w in range(self.W):
+                self.keys[(w, cl)] = wl.micro_keys(c, w, cl, self.device).to(torch.int32)
+        g = torch.Generator(device=self.device).manual_seed(c.seed + 5)
+        self.deltas = [torch.randn((c.batch, self.D), generator=g, device=self.device) * c.delta_std
+                       for _ in range(self.W)]
+        self.out = torch.empty((c.batch, self.D), device=self.device)
+
+    def start(self, pm):
+        for w in range(self.W):
+            for j in range(self.lookahead):
+                pm.intent(w, self.keys[(w, j)], j, j + self.span)
+
+    def step(self, pm, cl):
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, self.keys[(w, j)], j, j + self.span)
+            k = self.keys[(w, cl)]
+            pm.pull(w, k, out=self.out)
+            pm.push(w, k, self.deltas[w])
+            pm.advance_clock(w)
+        pm.sync()
+
+    def keys_per_step(self):
+        return 2 * self.W * self.cfg.batch     # pulled + pushed
+
+    # host-buffer variant for the end-to-end number
+    def prepare_host(self, clocks):
+        self.hkeys = {(w, c): self.keys[(w, c)].cpu().pin_memory() for c in clocks
+                      for w in range(self.W) if (w, c) in self.keys}
+        self.hdeltas = [d.cpu().pin_memory() for d in self.deltas]
+        self.hout = torch.empty((self.cfg.batch, self.D), pin_memory=True)
+
+    def step_host(self, pm, cl):
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, self.hkeys[(w, j)], j, j + self.span)
+            k = self.hkeys[(w, cl)]
+            pm.pull(w, k, out=self.hout)
+            pm.push(w, k, self.hdeltas[w])
+            pm.advance_clock(w)
+        pm.sync()
+
+    def host_bytes_per_step(self):
+        b = self.cfg.batch
+        h2d = self.W * (b * 4 * 3 + b * self.D * 4)   # intent keys, pull keys, push keys, deltas
+        d2h = self.W * b * self.D * 4                  # pulled rows
+        return h2d, d2h
+
+
+class MF:
+    """Matrix factorisation 10M x 1M, rank 100 + AdaGrad: fused MF step per worker per clock."""
+
+    def __init__(self, args, device, cfg=None):
+        self.cfg = cfg or wl.MF
+        c = self.cfg
+        self.device = device
+        self.K, self.D, self.W = c.num_keys, c.value_len, c.workers
+        self.lookahead, self.span = c.lookahead, c.span
+        self.row = self.D * 4
+        self.capacity = min(self.W * 2 * (self.lookahead + 1) * 2 * c.batch, 80_000_000)
+        self.samples_per_step = self.W * c.batch
+
+    def config(self):
+        c = self.cfg
+        return {"workload": c.name, "rows": c.rows, "cols": c.cols, "rank": c.rank,
+                "adagrad": c.adagrad, "workers": c.workers, "batch_per_worker": c.batch,
+                "zipf_s": c.zipf_s, "lookahead": c.lookahead, "intent_span": c.span, "lr": c.lr}
+
+    def init_store(self):
+        c = self.cfg
+        return hashgen.init_store_torch(self.K, self.D, c.rank, c.seed, c.init_std, self.device,
+                                        chunk_rows=1 << 21)
+
+    def prepare(self, clocks):
+        c = self.cfg
+        self.data = {}
+        for cl in range(clocks + self.lookahead + 1):
+            for w in range(self.W):
+                r, co, v = wl.mf_batch(c, w, cl, self.device)
+                self.data[(w, cl)] = (r.to(torch.int32), co.to(torch.int32), v,
+                                      torch.cat([r, co]).to(torch.int32))
+        self.loss = torch.zeros(self.W, dtype=torch.float64, device=self.device)
+
+    def start(self, pm):
+        for w in range(self.W):
+            for j in range(self.lookahead):
+                pm.intent(w, self.data[(w, j)][3], j, j + self.span)
+
+    def step(self, pm, cl, data=None):
+        c = self.cfg
+        data = data or self.data
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, data[(w, j)][3], j, j + self.span)
+            r, co, v, _ = data[(w, cl)]
+            pm.mf_step(w, r, co, v, c.rank, c.adagrad, c.lr, c.eps, loss_out=self.loss[w:w + 1])
+            pm.advance_clock(w)
+        pm.sync()
+
+    def keys_per_step(self):
+        return 4 * self.W * self.cfg.batch     # 2 rows read + 2 delta rows written per cell
+
+    def step_alg_bytes(self):
+        # per cell: keys + value in (12 B), 2 rows read, 2 delta rows + 2 keys written
+        return self.W * self.cfg.batch * (12 + 4 * self.row + 8)
+
+    def prepare_host(self, clocks):
+        self.hdata = {(w, c): tuple(x.cpu().pin_memory() for x in self.data[(w, c)]) for c in clocks
+                      for w in range(self.W) if (w, c) in self.data}
+        self.hloss = torch.zeros(1, dtype=torch.float64, pin_memory=True)
+
+    def step_host(self, pm, cl):
+        c = self.cfg
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, self.hdata[(w, j)][3], j, j + self.span)
+            r, co, v, _ = self.hdata[(w, cl)]
+            pm.mf_step(w, r, co, v, c.rank, c.adagrad, c.lr, c.eps, loss_out=self.hloss)
+            pm.advance_clock(w)
+        pm.sync()
+
+    def host_bytes_per_step(self):
+        b = self.cfg.batch
+        h2d = self.W * (b * 8 + b * 4 + 2 * b * 4)    # rows+cols, values, intent keys
+        d2h = self.W * 8                               # batch loss
+        return h2d, d2h
+
+
+WORKLOADS = {"micro": Micro, "mf": MF}
+
+
+# ---------------------------------------------------------------------------
+# algorithmic bytes: the minimum each operation must move (keys 4 B, row D*4 B)
+# ---------------------------------------------------------------------------
+def alg_bytes_per_step(wk, d, steps):
+    """d: differences of the library counters over `steps` profiled steps."""
+    row = wk.row
+    per = {k: v / steps for k, v in d.items()}
+    R, U = per["push_rows"], per["push_unique"]
+    out = {
+        # read keys + scatter rows, and one row read per distinct key (+ its slot)
+        "push": R * (4 + row) + U * (4 + 4 * row),
+        # the scatter kernel alone also reads the sorted (key, position) pairs
+        "push_kernel": R * (8 + row) + U * (4 + 4 * row),
+        # main += pending (2 rows per key); val := main, pending := 0 (3 rows per replica)
+        "sync": per["sync_keys"] * 2 * row + per["sync_replicas"] * 3 * row,
+        # destroy: read pending, read+write main; create: read main, write val and pending
+        "advance": (per["created"] + per["destroyed"]) * 3 * row,
+    }
+    if isinstance(wk, Micro):
+        B, W = wk.cfg.batch, wk.W
+        out["pull"] = W * B * (4 + row) + U * (4 + row)
+        out["pull_kernel"] = out["pull"]
+        out["intent"] = W * B * 4 + U * 4
+    else:
+        out["step"] = wk.step_alg_bytes()
+        out["intent"] = R * 4 + U * 4
+    return out
+
+
+COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "created", "destroyed")
+
+
+def run_ours(args, ws, rank, local):
+    from paper_2206_00470_gb300 import adapm
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    wk = WORKLOADS[args.workload](args, device)
+    total_clocks = args.warmup + args.steps
+    t0 = time.time()
+    wk.prepare(total_clocks + 2 * args.steps + 2)
+    init = wk.init_store()
+    pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init)
+    del init
+    torch.cuda.synchronize()
+    setup_s = time.time() - t0
+
+    # -- device-resident run ---------------------------------------------------
+    wk.start(pm)
+    for cl in range(args.warmup):
+        wk.step(pm, cl)
+    pm.wait()
+    clocks = ClockSampler(local)
+    start_ev, end_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(ws)
+    torch.cuda.synchronize()
+    l0 = adapm.kernel_launches()
+    clocks.start()
+    start_ev.record()
+    for cl in range(args.warmup, total_clocks):
+        wk.step(pm, cl)
+    end_ev.record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    launches = adapm.kernel_launches() - l0
+    barrier(ws)
+    ms = start_ev.elapsed_time(end_ev)
+    pm.wait()
+    stats = pm.stats()
+
+    # -- per-operation device times (library events), same steps again ---------
+    s0 = pm.stats()
+    pm.profile_enable(True)
+    pm.profile_read()
+    for cl in range(total_clocks, total_clocks + args.steps):
+        wk.step(pm, cl)
+    prof = pm.profile_read()
+    pm.profile_enable(False)
+    s1 = pm.stats()
+    pm.wait()
+
+    # -- end to end through the C ABI with pinned host buffers -------------------
+    e2e_ms = None
+    if not args.no_e2e:
+        base = total_clocks + args.steps
+        wk.prepare_host(range(base, base + 1 + args.steps + wk.lookahead + 1))
+        wk.step_host(pm, base)
+        pm.wait()
+        barrier(ws)
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        for cl in range(base + 1, base + 1 + args.steps):
+            wk.step_host(pm, cl)
+        pm.wait()
+        e2e_ms = (time.perf_counter() - t) * 1e3
+        barrier(ws)
+    pm.close()
+
+    ms_max = max_over_ranks(ms, ws, device)
+    keys_total = sum_over_ranks(wk.keys_per_step() * args.steps, ws, device)
+    value = keys_total / (ms_max / 1e3)
+    samples = sum_over_ranks(wk.samples_per_step * args.steps, ws, device) / (ms_max / 1e3)
+    peak, peak_src = load_peaks()
+
+    steps = args.steps
+    alg = alg_bytes_per_step(wk, {k: s1[k] - s0[k] for k in COUNTERS}, steps)
+    ops = {}
+    for name, (t_ms, calls) in prof.items():
+        if calls == 0:
+            continue
+        d = {"ms_per_step": t_ms / steps, "calls_per_step": calls / steps}
+        if name in alg and t_ms > 0:
+            gbs = alg[name] / (t_ms / steps / 1e3) / 1e9
+            d["alg_bytes_per_step"] = alg[name]
+            d["alg_GBps"] = gbs
+            d["frac_of_peak"] = gbs / peak
+        ops[name] = d
+
+    # dominant kernel: the library kernel (or fused kernel pair) with the largest time
+    roofline = None
+    cand = [(ops[n]["ms_per_step"], n) for n in ("push_kernel", "pull_kernel", "sync", "step")
+            if n in ops and n in alg]
+    if cand:
+        t_ms, name = max(cand)
+        calls = ops[name]["calls_per_step"]
+        a = alg[name] / calls
+        dur = t_ms / calls / 1e3
+        ach = a / dur / 1e9
+        roofline = {"bound": "hbm", "kernel": name, "achieved": ach, "peak": peak,
+                    "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
+                    "traffic": None, "alg_bytes_per_launch": a, "launch_ms": t_ms / calls}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "samples_per_s": samples if wk.samples_per_step else None,
+        "config": dict(wk.config(), parallelism=f"replicas{ws}",
+                       l2="inputs larger than L2 (no flush)"),
+        "gpu_launches": int(launches),
+        "clocks": clk,
+        "roofline": roofline,
+        "ops": ops,
+        "stats": {k: stats[k] for k in ("live_replicas", "high_water", "capacity")},
+        "setup_s": setup_s,
+    }
+    if e2e_ms is not None:
+        e2e_max = max_over_ranks(e2e_ms, ws, device)
+        h2d, d2h = wk.host_bytes_per_step()
+        line["e2e"] = {"value": keys_total / (e2e_max / 1e3), "unit": UNIT,
+                       "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    return line
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (reported baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(workload, budget_s, args):
+    """Time the CPU oracle on a bounded sample of the workload; returns (keys/s, samples/s, desc)."""
+    from oracle import ParameterManagerOracle, steps as osteps
+    from oracle import driver as odriver
+    import dataclasses
+    if workload == "micro":
+        base = wl.MICRO
+        cfg = dataclasses.replace(base, batch=1 << 13,
+                                  zipf_s=args.zipf if args.zipf is not None else base.zipf_s,
+                                  span=args.span or base.span)
+        nclk = 24
+        kmap = {}
+        for cl in range(nclk + cfg.lookahead + 1):
+            for w in range(cfg.workers):
+                kmap[(w, cl)] = wl.micro_keys(cfg, w, cl, "cpu").numpy()
+        touched = np.unique(np.concatenate(list(kmap.values())))
+        rel = {k: np.searchsorted(touched, v) for k, v in kmap.items()}
+        init = hashgen.init_rows_np(touched, cfg.value_len, cfg.value_len, cfg.seed, cfg.init_std)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+        g = np.random.default_rng(0)
+        deltas = (g.standard_normal((cfg.batch, cfg.value_len)) * cfg.delta_std).astype(np.float32)
+
+        def work(w, cl):
+            k = rel[(w, cl)]
+            pm.pull(w, k)
+            pm.push(w, k, deltas)
+
+        keys_of = lambda w, cl: rel[(w, cl)]  # noqa: E731
+        odriver.start(pm, cfg.workers, cfg.lookahead, cfg.span, keys_of)
+        t = time.perf_counter()
+        done = 0
+        while done < nclk and time.perf_counter() - t < budget_s:
+            odriver.clock(pm, cfg.workers, cfg.lookahead, cfg.span, done, keys_of, work)
+            done += 1
+        el = time.perf_counter() - t
+        keys = done * cfg.workers * cfg.batch * 2
+        desc = (f"{done} clocks of {cfg.workers} workers x {cfg.batch} Zipf({cfg.zipf_s}) keys of the "
+                f"100M-key x 64 workload (store restricted to the {touched.size} touched keys)")
+        return keys / el, None, desc
+    if workload == "mf":
+        cfg = dataclasses.replace(wl.MF, batch=2048)
+        nclk = 24
+        data = {}
+        for cl in range(nclk + cfg.lookahead + 1):
+            for w in range(cfg.workers):
+                r, co, v = wl.mf_batch(cfg, w, cl, "cpu")
+                data[(w, cl)] = (r.numpy(), co.numpy(), v.numpy())
+        touched = np.unique(np.concatenate([np.concatenate([a, b]) for a, b, _ in data.values()]))
+        rel = {k: (np.searchsorted(touched, a), np.searchsorted(touched, b), v)
+               for k, (a, b, v) in data.items()}
+        init = hashgen.init_rows_np(touched, cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+
+        def work(w, cl):
+            a, b, v = rel[(w, cl)]
+            return osteps.mf_step(pm, w, a, b, v, cfg.rank, cfg.lr, cfg.adagrad, cfg.eps)
+
+        keys_of = lambda w, cl: np.concatenate(rel[(w, cl)][:2])  # noqa: E731
+        odriver.start(pm, cfg.workers, cfg.lookahead, cfg.span, keys_of)
+        t = time.perf_counter()
+        done = 0
+        while done < nclk and time.perf_counter() - t < budget_s:
+            odriver.clock(pm, cfg.workers, cfg.lookahead, cfg.span, done, keys_of, work)
+            done += 1
+        el = time.perf_counter() - t
+        cells = done * cfg.workers * cfg.batch
+        desc = (f"{done} clocks of {cfg.workers} workers x {cfg.batch} cells of the 10M x 1M rank-100 "
+                f"AdaGrad workload (store restricted to the {touched.size} touched keys)")
+        return 4 * cells / el, cells / el, desc
+    raise ValueError(workload)
+
+
+def cpu_baseline(args):
+    threads = torch.get_num_threads()
+    v, s, desc = oracle_sample(args.workload, args.cpu_budget, args)
+    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
+            "samples_per_s": s, "host_threads_available": threads}
+
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return None
+    base = cpu_baseline(args)
+    t_steps = []
+    for _ in range(args.steps):
+        t_steps.append(base["value"])
+    line = {
+        "impl": "reference", "metric": METRIC, "value": base["value"], "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": dict(WORKLOADS[args.workload](args, None).config(), parallelism="replicas1",
+                       reference="CPU oracle (plain Python/numpy, 1 core)"),
+        "cpu_baseline": base,
+        "e2e": {"value": base["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    return line
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="micro", choices=sorted(WORKLOADS))
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--zipf", type=float, default=None)
+    ap.add_argument("--span", type=int, default=None)
+    ap.add_argument("--keys", type=int, default=None, help="micro: key-space size (default 1e8)")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        if ws > 1:
+            init_dist(ws, "gloo")
+        line = run_reference(args, ws, rank)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    init_dist(ws, "nccl")
+    # the oracle baseline runs on the host before any CUDA work (rank 0, N=1 only)
+    base = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        base = cpu_baseline(args)
+    line = run_ours(args, ws, rank, local)
+    if rank == 0:
+        line["cpu_baseline"] = base
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

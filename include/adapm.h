@@ -180,6 +180,10 @@ typedef struct {
   uint64_t capacity;
   uint64_t created, destroyed;
   uint64_t last_push_unique; /* distinct keys of the last push */
+  uint64_t push_rows;        /* rows pushed, cumulative (training steps included) */
+  uint64_t push_unique;      /* distinct keys per push, summed over pushes */
+  uint64_t sync_keys;        /* keys merged by sync, cumulative */
+  uint64_t sync_replicas;    /* replicas refreshed by sync, cumulative */
 } adapm_stats;
 
 adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);
@@ -193,6 +197,10 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);
 #define ADAPM_NUM_OPS 8
 adapm_status adapm_profile_enable(adapm_ctx* ctx, int enable);
 adapm_status adapm_profile_read(adapm_ctx* ctx, double* ms_out, uint64_t* calls_out);
+
+/* Number of CUDA kernels this library has launched in this process (all
+ * contexts), for checking which work ran on the GPU. */
+adapm_status adapm_kernel_launches(uint64_t* out);
 
 /* Message for the last error returned on this context ("" if none). */
 const char* adapm_last_error(adapm_ctx* ctx);

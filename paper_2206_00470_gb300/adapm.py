@@ -26,7 +26,7 @@ EXPORTS = [
     "adapm_push", "adapm_sync", "adapm_wait", "adapm_mf_step", "adapm_complex_step",
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
     "adapm_refcounts", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
-    "adapm_profile_read", "adapm_last_error",
+    "adapm_profile_read", "adapm_kernel_launches", "adapm_last_error",
 ]
 
 
@@ -49,6 +49,10 @@ class Stats(ctypes.Structure):
         ("created", ctypes.c_uint64),
         ("destroyed", ctypes.c_uint64),
         ("last_push_unique", ctypes.c_uint64),
+        ("push_rows", ctypes.c_uint64),
+        ("push_unique", ctypes.c_uint64),
+        ("sync_keys", ctypes.c_uint64),
+        ("sync_replicas", ctypes.c_uint64),
     ]
 
 
@@ -91,6 +95,7 @@ def load(path=LIB_PATH):
         "adapm_get_stats": [P, ctypes.POINTER(Stats)],
         "adapm_profile_enable": [P, I],
         "adapm_profile_read": [P, P, P],
+        "adapm_kernel_launches": [ctypes.POINTER(U64)],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -100,6 +105,15 @@ def load(path=LIB_PATH):
     L.adapm_last_error.restype = ctypes.c_char_p
     _lib = L
     return L
+
+
+def kernel_launches():
+    """Kernels launched by libadapm in this process so far."""
+    v = ctypes.c_uint64()
+    st = load().adapm_kernel_launches(ctypes.byref(v))
+    if st != OK:
+        raise AdaPMError(st, "adapm_kernel_launches")
+    return v.value
 
 
 def _torch():

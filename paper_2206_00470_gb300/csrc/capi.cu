@@ -5,6 +5,7 @@
 // stream; scratch comes from a context-owned stream-ordered memory pool.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -19,6 +20,12 @@
 #include "store_launch.cuh"
 
 using namespace adapm;
+
+namespace {
+std::atomic<unsigned long long> g_launches{0};
+}  // namespace
+
+void adapm::note_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 namespace {
 
@@ -51,6 +58,7 @@ struct adapm_ctx {
   int64_t next_list = 0;
   std::string err;
   bool broken = false;
+  uint64_t push_rows_host = 0;
   bool prof = false;
   std::vector<std::tuple<int, cudaEvent_t, cudaEvent_t>> pending;
   std::vector<cudaEvent_t> spare_events;
@@ -227,15 +235,20 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   launch_prep_keys(dkeys, n, ctx->s.K, ka, ctx->dstate, allow_nokey, ctx->sms, ctx->stream);
   uint32_t *sk = nullptr, *sp = nullptr;
   radix_sort(ka, kb, va, vb, true, true, n, ctx->bits, hist, ctx->stream, &sk, &sp);
-  // chunks: enough for every SM to hold many groups, at least 16 rows each
-  uint64_t chunk = 16;
-  while (chunk < 128 && n / (chunk * 2) >= (uint64_t)ctx->sms * 128) chunk *= 2;
+  const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
-  float *ph = nullptr, *pt = nullptr;
+  const uint64_t nspans = push_spans(ctx->s.D, n, chunk);
+  float *ph = nullptr, *pt = nullptr, *bh = nullptr, *bt = nullptr;
+  uint32_t* longs = nullptr;
   CK(pool_alloc(ctx, &ph, nchunks * ctx->s.D));
   CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
+  CK(pool_alloc(ctx, &bh, nspans * ctx->s.D));
+  CK(pool_alloc(ctx, &bt, nspans * ctx->s.D));
+  CK(pool_alloc(ctx, &longs, nspans / 8 + 2));
+  CK(cudaMemsetAsync(longs, 0, sizeof(uint32_t), ctx->stream));
   CK(cudaMemsetAsync(&ctx->dstate->last_unique, 0, sizeof(uint32_t), ctx->stream));
-  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w};
+  ctx->push_rows_host += n;
+  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, bh, bt, longs + 1, longs};
   {
     ProfScope ps(ctx, 6);
     launch_push(ctx->s, a, ctx->sms, ctx->stream);
@@ -247,6 +260,9 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   pool_free(ctx, hist);
   pool_free(ctx, ph);
   pool_free(ctx, pt);
+  pool_free(ctx, bh);
+  pool_free(ctx, bt);
+  pool_free(ctx, longs);
   return check_launch(ctx, "push");
 }
 
@@ -742,6 +758,10 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
   out->created = h.created;
   out->destroyed = h.destroyed;
   out->last_push_unique = h.last_unique;
+  out->push_rows = ctx->push_rows_host;
+  out->push_unique = h.push_unique;
+  out->sync_keys = h.sync_keys;
+  out->sync_replicas = h.sync_replicas;
   return ADAPM_OK;
 }
 
@@ -772,6 +792,12 @@ adapm_status adapm_profile_read(adapm_ctx* ctx, double* ms_out, uint64_t* calls_
     ctx->prof_ms[i] = 0;
     ctx->prof_calls[i] = 0;
   }
+  return ADAPM_OK;
+}
+
+adapm_status adapm_kernel_launches(uint64_t* out) {
+  if (!out) return ADAPM_EINVAL;
+  *out = g_launches.load(std::memory_order_relaxed);
   return ADAPM_OK;
 }
 

@@ -41,6 +41,10 @@ struct DevState {
   unsigned long long destroyed;
   int32_t live;
   int32_t pad;
+  unsigned long long push_rows;       // rows pushed (cumulative)
+  unsigned long long push_unique;     // distinct keys over all pushes (cumulative)
+  unsigned long long sync_keys;       // keys merged by sync (cumulative)
+  unsigned long long sync_replicas;   // replicas refreshed by sync (cumulative)
 };
 
 // Plain view of the device state passed to kernels by value.
@@ -87,5 +91,8 @@ void compact_replica_keys(const int32_t* map_w, uint64_t K, uint32_t* out, uint3
                           uint32_t* tmp, cudaStream_t stream);
 
 int bits_for(uint64_t num_keys);   // bits covering [0, K] (K itself is the sentinel range)
+
+// Process-wide count of kernels launched by the library (capi.cu).
+void note_launches(uint64_t n);
 
 }  // namespace adapm

@@ -248,6 +248,7 @@ void compact(Sel sel, uint32_t* out, uint32_t* count, uint32_t* tmp, cudaStream_
     cudaMemsetAsync(count, 0, sizeof(uint32_t), stream);
     return;
   }
+  note_launches(3);
   compact_count_kernel<Sel><<<nb, kSortThreads, 0, stream>>>(sel, tmp);
   scan_tiles_kernel<<<1, 1024, 0, stream>>>(tmp, nb, count);
   compact_write_kernel<Sel><<<nb, kSortThreads, 0, stream>>>(sel, tmp, out);
@@ -283,6 +284,7 @@ void radix_sort(uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, bool wit
   for (int p = 0; p < passes; ++p) {
     const int b = per < bits - shift ? per : bits - shift;
     const uint32_t mask = (1u << b) - 1u;
+    note_launches(3);
     radix_hist_kernel<<<nb, kSortThreads, 0, stream>>>(kin, n, shift, mask, hist, nb);
     radix_scan_kernel<<<mask + 1, kSortThreads, 0, stream>>>(hist, nb, totals);
     if (!with_vals) {

@@ -400,6 +400,7 @@ void launch_mf_step(const Store& s, uint32_t w, const uint32_t* rows, const uint
                     const float* vals, uint64_t n, uint32_t dim, bool adagrad, float lr, float eps,
                     const StepOut& o, int sms, cudaStream_t stream) {
   const unsigned grid = o.loss_blocks;
+  note_launches(1);
   const uint32_t dim4 = dim / 4;
   const int a = adagrad ? 1 : 0;
   if (dim4 <= 4) mf_step_kernel<4, 1><<<grid, kThreads, 0, stream>>>(s, w, rows, cols, vals, n, dim, a, lr, eps, o);
@@ -415,6 +416,7 @@ void launch_complex_step(const Store& s, uint32_t w, const uint32_t* heads, cons
                          uint32_t dim, float lr, float eps, const StepOut& o, int sms,
                          cudaStream_t stream) {
   const unsigned grid = o.loss_blocks;
+  note_launches(1);
   const uint32_t h4 = dim / 8;
   if (h4 <= 32) complex_step_kernel<1, 4><<<grid, kThreads, 0, stream>>>(s, w, heads, rels, tails, negs, n, n_neg, dim, lr, eps, o);
   else complex_step_kernel<2, 2><<<grid, kThreads, 0, stream>>>(s, w, heads, rels, tails, negs, n, n_neg, dim, lr, eps, o);
@@ -425,6 +427,7 @@ void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const
                       uint32_t vocab, uint32_t dim, float lr, const StepOut& o, int sms,
                       cudaStream_t stream) {
   const unsigned grid = o.loss_blocks;
+  note_launches(1);
   const uint32_t D4 = dim / 4;
   if (D4 <= 32) sgns_step_kernel<1, 8><<<grid, kThreads, 0, stream>>>(s, w, centres, contexts, negs, n, n_ctx, n_neg, vocab, lr, o);
   else if (D4 <= 64) sgns_step_kernel<2, 4><<<grid, kThreads, 0, stream>>>(s, w, centres, contexts, negs, n, n_ctx, n_neg, vocab, lr, o);
@@ -433,6 +436,7 @@ void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const
 }
 
 void launch_loss_reduce(const double* part, unsigned nparts, double* out, cudaStream_t stream) {
+  note_launches(1);
   loss_reduce_kernel<<<1, 32, 0, stream>>>(part, nparts, out);
 }
 

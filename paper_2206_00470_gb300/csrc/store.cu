@@ -131,10 +131,44 @@ __device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, u
   }
 }
 
+// tot += rows first..last of a piece array (ascending, loads issued in batches)
+template <int G, int C>
+__device__ __forceinline__ void sum_pieces(float4 (&tot)[C], const float4* pieces, uint64_t first,
+                                           uint64_t last, uint32_t D4, int lane) {
+  constexpr int UB = 8 / C > 0 ? 8 / C : 1;
+  for (uint64_t m0 = first; m0 <= last; m0 += UB) {
+    float4 t[UB][C];
+#pragma unroll
+    for (int u = 0; u < UB; ++u)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        t[u][c] = (m0 + u <= last && col < D4) ? pieces[(m0 + u) * D4 + col] : f4zero();
+      }
+#pragma unroll
+    for (int u = 0; u < UB; ++u)
+      if (m0 + u <= last)
+#pragma unroll
+        for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+  }
+}
+
+// Each block stages kPushSpan consecutive sorted positions (keys and source
+// positions) in shared memory; its groups own consecutive chunks of them.
+constexpr int kPushSpan = 1024;
+// a segment cut by chunk boundaries and spanning at most this many further
+// chunks is combined by one group; longer ones (hot keys) by a whole block
+constexpr int kShortSpan = 8;
+
 template <int G, int C, int R>
-__global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs a) {
+__global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 3) push_chunks_kernel(Store s, PushArgs a) {
+  constexpr int NG = kThreads / G;
+  const uint32_t CH = (uint32_t)a.chunk;            // rows per group, NG * CH <= kPushSpan
+  const uint32_t span = NG * CH;
+  __shared__ uint32_t sk[kPushSpan + 2];   // sk[0]: key before the span; sk[1+len]: key after it
+  __shared__ uint32_t sp[kPushSpan];
   const int lane = threadIdx.x & (G - 1);
-  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const int gi = threadIdx.x / G;
   const uint32_t D4 = s.D >> 2;
   const float4* d4 = reinterpret_cast<const float4*>(a.deltas);
   float4* val4 = reinterpret_cast<float4*>(s.val);
@@ -144,37 +178,39 @@ __global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs
   float4* pt4 = reinterpret_cast<float4*>(a.part_tail);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   uint32_t heads = 0;
-  for (uint64_t j = g; j < a.nchunks; j += ng) {
-    const uint64_t p0 = j * a.chunk;
-    const uint64_t p1 = p0 + a.chunk < a.n ? p0 + a.chunk : a.n;
-    const bool has_prev = p0 > 0;
-    const uint32_t prev_key = has_prev ? a.skeys[p0 - 1] : 0u;
-    const bool has_after = p1 < a.n;
-    const uint32_t after_key = has_after ? a.skeys[p1] : 0u;
+  for (uint64_t P0 = (uint64_t)blockIdx.x * span; P0 < a.n; P0 += (uint64_t)gridDim.x * span) {
+    const uint32_t len = (uint32_t)(a.n - P0 < (uint64_t)span ? a.n - P0 : span);
+    __syncthreads();
+    for (uint32_t i = threadIdx.x; i < len; i += kThreads) {
+      sk[1 + i] = a.skeys[P0 + i];
+      sp[i] = a.spos[P0 + i];
+    }
+    if (threadIdx.x == 0) {
+      sk[0] = P0 > 0 ? a.skeys[P0 - 1] : kNoKey;
+      sk[1 + len] = P0 + len < a.n ? a.skeys[P0 + len] : kNoKey;
+    }
+    __syncthreads();
+    const uint32_t p0 = gi * CH;
+    const uint32_t p1 = p0 + CH < len ? p0 + CH : len;
+    const uint64_t j = P0 / CH + gi;                 // global chunk index
+    const bool has_prev = P0 + p0 > 0;
     uint32_t cur = 0;
     bool cur_valid = false, cur_started = false;
     float4 run[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) run[c] = f4zero();
-    for (uint64_t p = p0; p < p1; p += R) {
-      uint32_t k[R], src[R];
-#pragma unroll
-      for (int r = 0; r < R; ++r) {
-        const bool v = p + r < p1;
-        k[r] = v ? a.skeys[p + r] : kNoKey;
-        src[r] = v ? a.spos[p + r] : 0u;
-      }
-      const bool q_in = p + R < p1;
-      const uint32_t knext = q_in ? a.skeys[p + R] : after_key;
-      const bool knext_valid = q_in || has_after;
+    for (uint32_t p = p0; p < p1; p += R) {
+      uint32_t k[R];
       float4 d[R][C];
 #pragma unroll
       for (int r = 0; r < R; ++r) {
+        const bool v = p + r < p1;
+        k[r] = v ? sk[1 + p + r] : kNoKey;
+        const uint32_t src = v ? sp[p + r] : 0u;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          d[r][c] = (p + r < p1 && k[r] != kNoKey && col < D4)
-                        ? __ldg(d4 + (uint64_t)src[r] * D4 + col) : f4zero();
+          d[r][c] = (v && k[r] != kNoKey && col < D4) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
         }
       }
       uint32_t fl[R];   // bit0 piece ends here, bit1 piece started in chunk, bit2 segment ends here
@@ -185,7 +221,7 @@ __global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs
           if (!cur_valid || k[r] != cur) {
             cur = k[r];
             cur_valid = true;
-            cur_started = (p + r > p0) || !has_prev || prev_key != k[r];
+            cur_started = (p + r > p0) || !has_prev || sk[p0] != k[r];
             if (cur_started && k[r] != kNoKey) ++heads;
 #pragma unroll
             for (int c = 0; c < C; ++c) run[c] = f4zero();
@@ -195,17 +231,10 @@ __global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs
             run[c] = f4add(run[c], d[r][c]);
             d[r][c] = run[c];
           }
-          bool kn_valid;
-          uint32_t kn;
-          if (r + 1 < R && p + r + 1 < p1) {
-            kn = k[r + 1];
-            kn_valid = true;
-          } else {
-            kn = knext;
-            kn_valid = knext_valid;
-          }
-          const bool seg_end = !kn_valid || kn != k[r];
-          const bool last = (p + r + 1 == p1);
+          const uint32_t nxt = p + r + 1;             // local position of the next row
+          const bool kn_valid = P0 + nxt < a.n;
+          const bool seg_end = !kn_valid || sk[1 + nxt] != k[r];
+          const bool last = nxt == p1;
           fl[r] = ((seg_end || last) ? 1u : 0u) | (cur_started ? 2u : 0u) | (seg_end ? 4u : 0u);
           if (k[r] == kNoKey) fl[r] = 0;
         }
@@ -251,14 +280,86 @@ __global__ void __launch_bounds__(kThreads) push_chunks_kernel(Store s, PushArgs
         }
       }
     }
+    // combine the chunk pieces inside this span: a segment begun in chunk gi
+    // that ends later in the span is applied here; one that leaves the span
+    // leaves a span tail piece, and the span's first segment, begun before
+    // the span, a span head piece (both combined across spans by the fix-up)
+    __syncthreads();
+    const uint64_t b = P0 / span;
+    const uint64_t jb = P0 / CH;
+    if (p0 < p1) {
+      const uint32_t kl = sk[1 + p1 - 1];
+      const bool started = (P0 + p0 == 0) || sk[p0] != kl;
+      const bool cont = (P0 + p1 < a.n) && sk[1 + p1] == kl;
+      if (kl != kNoKey && started && cont) {
+        uint32_t q = p1, g_last = gi;
+        bool leaves = false;
+        while (true) {
+          if (q == len) {
+            leaves = true;
+            break;
+          }
+          ++g_last;
+          const uint32_t qe = q + CH < len ? q + CH : len;
+          if (P0 + qe < a.n && sk[1 + qe] == kl) {
+            q = qe;
+            continue;
+          }
+          break;
+        }
+        float4 tot[C];
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          tot[c] = col < D4 ? pt4[(jb + gi) * D4 + col] : f4zero();
+        }
+        sum_pieces<G, C>(tot, ph4, jb + gi + 1, jb + g_last, D4, lane);
+        if (leaves) {
+          float4* bt4 = reinterpret_cast<float4*>(a.span_tail);
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            if (col < D4) bt4[b * D4 + col] = tot[c];
+          }
+        } else {
+          apply_sum<C>(s, mapw, kl, tot, lane, G);
+        }
+      }
+    }
+    if (gi == 0 && P0 > 0 && sk[1] == sk[0] && sk[1] != kNoKey) {
+      const uint32_t kf = sk[1];
+      uint32_t g_last = 0;
+      uint32_t qe = CH < len ? CH : len;
+      while (qe < len && P0 + qe < a.n && sk[1 + qe] == kf) {
+        ++g_last;
+        qe = qe + CH < len ? qe + CH : len;
+      }
+      float4 tot[C];
+#pragma unroll
+      for (int c = 0; c < C; ++c) tot[c] = f4zero();
+      sum_pieces<G, C>(tot, ph4, jb, jb + g_last, D4, lane);
+      float4* bh4 = reinterpret_cast<float4*>(a.span_head);
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) bh4[b * D4 + col] = tot[c];
+      }
+    }
   }
-  if (lane == 0 && heads) atomicAdd(&s.st->last_unique, heads);
+  if (lane == 0 && heads) {
+    atomicAdd(&s.st->last_unique, heads);
+    atomicAdd(&s.st->push_unique, (unsigned long long)heads);
+  }
 }
 
-// A segment that starts in chunk j and continues past it is owned by j:
-// tail piece of j + head pieces of j+1 .. m_end, in chunk order.
+// A segment that starts in chunk j and continues past it is owned by j: its
+// sum is j's tail piece plus the head pieces of chunks j+1 .. m_end.  Spans
+// of at most kShortSpan further chunks are combined here (loads issued
+// together); longer ones are listed for push_long_kernel.
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs a) {
+__global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs a, uint32_t* long_list,
+                                                              uint32_t* long_count) {
+  const uint64_t CH = a.chunk;
   const int lane = threadIdx.x & (G - 1);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   const uint32_t D4 = s.D >> 2;
@@ -266,42 +367,116 @@ __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs 
   const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   for (uint64_t j = g; j < a.nchunks; j += ng) {
-    const uint64_t p0 = j * a.chunk;
-    const uint64_t p1 = p0 + a.chunk;
+    const uint64_t p0 = j * CH;
+    const uint64_t p1 = p0 + CH;
     if (p1 >= a.n) continue;
     const uint32_t kl = a.skeys[p1 - 1];
     if (kl == kNoKey || a.skeys[p1] != kl) continue;
     if (p0 > 0 && a.skeys[p0 - 1] == kl) continue;           // started in an earlier chunk
-    // last chunk m whose first position still holds kl (monotone predicate)
-    uint64_t lo = j + 1, hi = a.nchunks - 1;
-    while (lo < hi) {
-      const uint64_t mid = (lo + hi + 1) / 2;
-      if (a.skeys[mid * a.chunk] == kl) lo = mid; else hi = mid - 1;
+    bool cont[kShortSpan];   // cont[t]: the segment continues past chunk j+1+t
+#pragma unroll
+    for (int t = 0; t < kShortSpan; ++t) {
+      const uint64_t e = (j + 2 + t) * CH;
+      cont[t] = e < a.n && a.skeys[e] == kl;
     }
-    const uint64_t m_end = lo;
+    int span = 0;            // further chunks after j+1 that the segment reaches
+#pragma unroll
+    for (int t = 0; t < kShortSpan; ++t)
+      if (span == t && cont[t]) ++span;
+    if (span == kShortSpan) {
+      if (lane == 0) long_list[atomicAdd(long_count, 1u)] = (uint32_t)j;
+      continue;
+    }
     float4 tot[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) {
       const uint32_t col = lane + c * G;
       tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
     }
-    constexpr int U = 8 / C > 0 ? 8 / C : 1;
-    for (uint64_t m = j + 1; m <= m_end; m += U) {
+    constexpr int UB = 8 / C > 0 ? 8 / C : 1;    // head pieces loaded together
+    for (int u0 = 0; u0 <= span; u0 += UB) {
+      float4 t[UB][C];
+#pragma unroll
+      for (int u = 0; u < UB; ++u)
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          t[u][c] = (u0 + u <= span && col < D4) ? ph4[(j + 1 + u0 + u) * D4 + col] : f4zero();
+        }
+#pragma unroll
+      for (int u = 0; u < UB; ++u)
+        if (u0 + u <= span)
+#pragma unroll
+          for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+    }
+    apply_sum<C>(s, mapw, kl, tot, lane, G);
+  }
+}
+
+// One block per long segment: its groups sum strided subsets of the head
+// pieces in increasing chunk order, then group 0 adds the tail piece and the
+// group sums in group order (a fixed summation tree: deterministic).
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a, const uint32_t* long_list,
+                                                             const uint32_t* long_count) {
+  constexpr int NG = kThreads / G;
+  const uint64_t CH = a.chunk;
+  __shared__ float4 part[NG][G * C];
+  __shared__ uint64_t s_mend;
+  const int lane = threadIdx.x & (G - 1);
+  const int gi = threadIdx.x / G;
+  const uint32_t D4 = s.D >> 2;
+  const float4* ph4 = reinterpret_cast<const float4*>(a.part_head);
+  const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
+  const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
+  const uint32_t nl = *long_count;
+  for (uint32_t e = blockIdx.x; e < nl; e += gridDim.x) {
+    const uint64_t j = long_list[e];
+    const uint32_t kl = a.skeys[(j + 1) * CH - 1];
+    if (threadIdx.x == 0) {
+      // last chunk m whose first position still holds kl (monotone predicate)
+      uint64_t lo = j + 1, hi = a.nchunks - 1;
+      while (lo < hi) {
+        const uint64_t mid = (lo + hi + 1) / 2;
+        if (a.skeys[mid * CH] == kl) lo = mid; else hi = mid - 1;
+      }
+      s_mend = lo;
+    }
+    __syncthreads();
+    const uint64_t m_end = s_mend;
+    float4 acc[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) acc[c] = f4zero();
+    constexpr int U = 4 / C > 0 ? 4 / C : 1;
+    for (uint64_t m = j + 1 + gi; m <= m_end; m += (uint64_t)NG * U) {
       float4 t[U][C];
 #pragma unroll
       for (int u = 0; u < U; ++u)
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          t[u][c] = (m + u <= m_end && col < D4) ? ph4[(m + u) * D4 + col] : f4zero();
+          const uint64_t mm = m + (uint64_t)u * NG;
+          t[u][c] = (mm <= m_end && col < D4) ? ph4[mm * D4 + col] : f4zero();
         }
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (m + u <= m_end)
 #pragma unroll
-          for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+        for (int c = 0; c < C; ++c) acc[c] = f4add(acc[c], t[u][c]);
     }
-    apply_sum<C>(s, mapw, kl, tot, lane, G);
+#pragma unroll
+    for (int c = 0; c < C; ++c) part[gi][lane + c * G] = acc[c];
+    __syncthreads();
+    if (gi == 0) {
+      float4 tot[C];
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
+        for (int q = 0; q < NG; ++q) tot[c] = f4add(tot[c], part[q][lane + c * G]);
+      }
+      apply_sum<C>(s, mapw, kl, tot, lane, G);
+    }
+    __syncthreads();
   }
 }
 
@@ -354,7 +529,8 @@ __global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restr
         }
         rcw[k] = (uint16_t)nw;
         create = old == 0 && nw > 0;
-        evict = old > 0 && nw == 0;
+        // a key whose replica was never created (capacity exhausted) has nothing to destroy
+        evict = old > 0 && nw == 0 && s.map[(uint64_t)w * s.K + k] >= 0;
       }
     }
     warp_append(create, k, &s.st->n_create, create_list);
@@ -362,56 +538,44 @@ __global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restr
   }
 }
 
-// evict: main[k] += acc[slot]; release slot
+// evict: main[k] += acc[slot]; the freed slot goes on the stack at
+// free_top + i (every listed key holds a replica), so no atomics are needed
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads) evict_kernel(Store s, uint32_t w, const uint32_t* __restrict__ list) {
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint32_t n = s.st->n_evict;
+  const int32_t top = s.st->free_top;
   int32_t* mapw = s.map + (uint64_t)w * s.K;
   float4* main4 = reinterpret_cast<float4*>(s.main);
   const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
-  constexpr int GPW = 32 / G;   // groups per warp
-  const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const uint64_t nwarps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
-  const int gi = (threadIdx.x & 31) / G;
-  for (uint64_t b = warp * GPW; b < n; b += nwarps * GPW) {
-    const uint64_t i = b + gi;
-    int32_t sl = -1;
-    uint32_t k = 0;
-    if (i < n) {
-      k = list[i];
-      sl = mapw[k];
-    }
-    if (sl >= 0) {
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  for (uint64_t i = g; i < n; i += ng) {
+    const uint32_t k = list[i];
+    const int32_t sl = mapw[k];
 #pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        if (col < D4) main4[(uint64_t)k * D4 + col] = f4add(main4[(uint64_t)k * D4 + col], acc4[(uint64_t)sl * D4 + col]);
-      }
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4) main4[(uint64_t)k * D4 + col] = f4add(main4[(uint64_t)k * D4 + col], acc4[(uint64_t)sl * D4 + col]);
     }
-    const bool rel = sl >= 0 && lane == 0;
-    const uint32_t m = __ballot_sync(0xFFFFFFFFu, rel);
-    if (m) {
-      const int leader = __ffs(m) - 1;
-      int32_t base = 0;
-      if ((int)(threadIdx.x & 31) == leader) {
-        base = atomicAdd(&s.st->free_top, (int32_t)__popc(m));
-        atomicSub(&s.st->live, (int32_t)__popc(m));
-        atomicAdd(&s.st->destroyed, (unsigned long long)__popc(m));
-      }
-      base = __shfl_sync(0xFFFFFFFFu, base, leader);
-      if (rel) {
-        mapw[k] = -1;
-        atomicAnd(s.holders + k, ~(1u << w));
-        s.slot_owner[sl] = kEmptySlot;
-        s.free_stack[base + __popc(m & lanemask_lt_())] = sl;
-      }
+    if (lane == 0) {
+      mapw[k] = -1;
+      atomicAnd(s.holders + k, ~(1u << w));
+      s.slot_owner[sl] = kEmptySlot;
+      s.free_stack[top + (int32_t)i] = sl;
     }
   }
 }
 
-__global__ void alloc_kernel(DevState* st) {
+// Single thread: account the evictions, then reserve the creations.  The
+// stack initially holds slots S-1 .. 0 (slot 0 on top) and positions below
+// S - high_water are never written, so popping down to alloc_base has used
+// every slot below S - alloc_base.
+__global__ void alloc_kernel(DevState* st, int32_t S) {
+  const uint32_t ne = st->n_evict;
+  st->free_top += (int32_t)ne;
+  st->live -= (int32_t)ne;
+  st->destroyed += ne;
   const uint32_t n = st->n_create;
   if ((int64_t)n > (int64_t)st->free_top) {
     st->errors |= ERR_NO_SLOTS;
@@ -424,6 +588,7 @@ __global__ void alloc_kernel(DevState* st) {
   st->n_create_ok = n;
   st->live += (int32_t)n;
   st->created += n;
+  if (S - st->alloc_base > st->high_water) st->high_water = S - st->alloc_base;
 }
 
 // create: val = main[k], acc = 0, take a slot from the stack
@@ -438,7 +603,6 @@ __global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, c
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  int32_t hw = 0;
   for (uint64_t i = g; i < n; i += ng) {
     const uint32_t k = list[i];
     // slots popped from the top of the stack: lowest free slots come first
@@ -455,10 +619,8 @@ __global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, c
       mapw[k] = sl;
       atomicOr(s.holders + k, 1u << w);
       s.slot_owner[sl] = ((unsigned long long)w << 32) | k;
-      hw = hw > sl + 1 ? hw : sl + 1;
     }
   }
-  if (lane == 0 && hw > 0) atomicMax(&s.st->high_water, hw);
 }
 
 // ---------------------------------------------------------------------------
@@ -473,6 +635,7 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
+  uint32_t nkeys = 0, nreps = 0;
   for (uint64_t sl = g; sl < hw; sl += ng) {
     const unsigned long long owner = s.slot_owner[sl];
     if (owner == kEmptySlot) continue;
@@ -480,6 +643,10 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
     const uint32_t k = (uint32_t)owner;
     const uint32_t mask = s.holders[k];
     if ((uint32_t)(__ffs(mask) - 1) != w) continue;   // the lowest holder merges
+    if (lane == 0) {
+      nkeys += 1;
+      nreps += (uint32_t)__popc(mask);
+    }
     float4 m[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) {
@@ -533,6 +700,10 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
         }
       }
     }
+  }
+  if (lane == 0 && nkeys) {
+    atomicAdd(&s.st->sync_keys, (unsigned long long)nkeys);
+    atomicAdd(&s.st->sync_replicas, (unsigned long long)nreps);
   }
 }
 
@@ -608,6 +779,7 @@ void launch_prep_keys(const uint32_t* in, uint64_t n, uint64_t K, uint32_t* out,
   if (n == 0) return;
   uint64_t b = (n + kThreads - 1) / kThreads;
   if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+  note_launches(1);
   prep_keys_kernel<<<(unsigned)b, kThreads, 0, stream>>>(in, n, K, out, st, allow_nokey ? 1 : 0);
 }
 
@@ -617,17 +789,50 @@ void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float*
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     constexpr int R = 8 / C > 0 ? 8 / C : 1;
+    note_launches(1);
     pull_kernel<G, C, R><<<grid_for((n + R - 1) / R, G, sms), kThreads, 0, stream>>>(s, w, keys, n, out);
   });
+}
+
+uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms) {
+  // longest chunk (<= kPushSpan / groups per block, >= 8) that still gives
+  // every SM four blocks of work
+  uint64_t ch = 0;
+  dispatch_gc(D / 4, [&](auto Gc, auto) {
+    constexpr int G = decltype(Gc)::value;
+    constexpr uint64_t NG = kThreads / G;
+    ch = kPushSpan / NG;
+    while (ch > 8 && n / (ch * NG) < (uint64_t)sms * 4) ch /= 2;
+  });
+  return ch;
+}
+
+uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk) {
+  uint64_t span = 0;
+  dispatch_gc(D / 4, [&](auto Gc, auto) {
+    constexpr int G = decltype(Gc)::value;
+    span = chunk * (kThreads / G);
+  });
+  return (n + span - 1) / span;
 }
 
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream) {
   if (a.n == 0) return;
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    constexpr int R = 8 / C > 0 ? 8 / C : 1;
-    push_chunks_kernel<G, C, R><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a);
-    push_fixup_kernel<G, C><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a);
+    constexpr int R = 4 / C > 0 ? 4 / C : 1;
+    uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
+    const uint64_t cap = (uint64_t)sms * 4;
+    note_launches(3);
+    push_chunks_kernel<G, C, R><<<(unsigned)(spans < cap ? spans : cap), kThreads, 0, stream>>>(s, a);
+    PushArgs sp = a;                       // the fix-up works on span pieces
+    sp.part_head = a.span_head;
+    sp.part_tail = a.span_tail;
+    sp.chunk = a.chunk * (kThreads / G);
+    sp.nchunks = spans;
+    push_fixup_kernel<G, C><<<grid_for(sp.nchunks, G, sms), kThreads, 0, stream>>>(s, sp, a.long_list,
+                                                                                  a.long_count);
+    push_long_kernel<G, C><<<(unsigned)sms, kThreads, 0, stream>>>(s, sp, a.long_list, a.long_count);
   });
 }
 
@@ -637,6 +842,7 @@ void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlist
     uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
     if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
     if (b == 0) continue;
+    note_launches(1);
     events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(lists[i].keys, lists[i].count,
                                                             lists[i].sign, s.ev_delta);
   }
@@ -644,6 +850,7 @@ void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlist
     uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
     if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
     if (b == 0) continue;
+    note_launches(1);
     events_apply_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, lists[i].keys, lists[i].count,
                                                               create_list, evict_list);
   }
@@ -655,8 +862,9 @@ void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     const unsigned grid = grid_for(max_events, G, sms);
+    note_launches(3);
     evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list);
-    alloc_kernel<<<1, 1, 0, stream>>>(s.st);
+    alloc_kernel<<<1, 1, 0, stream>>>(s.st, (int32_t)s.S);
     create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, create_list);
   });
 }
@@ -665,6 +873,7 @@ void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stre
   if (slot_bound == 0) return;
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    note_launches(1);
     sync_kernel<G, C><<<grid_for(slot_bound, G, sms), kThreads, 0, stream>>>(s);
   });
 }
@@ -672,6 +881,7 @@ void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stre
 void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, uint32_t* out,
                       cudaStream_t stream) {
   if (n == 0) return;
+  note_launches(1);
   refcounts_kernel<<<(unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, stream>>>(
       s, w, keys, n, out);
 }
@@ -679,6 +889,7 @@ void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t
 void launch_replica_rows(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, float* val,
                          float* acc, uint8_t* has, cudaStream_t stream) {
   if (n == 0) return;
+  note_launches(1);
   replica_rows_kernel<<<(unsigned)(n < 4096 ? n : 4096), 128, 0, stream>>>(s, w, keys, n, val, acc, has);
 }
 
@@ -686,6 +897,7 @@ void launch_init_pool(int32_t* free_stack, uint64_t S, unsigned long long* owner
   uint64_t b = (S + 255) / 256;
   if (b > 65535) b = 65535;
   if (b == 0) return;
+  note_launches(1);
   init_pool_kernel<<<(unsigned)b, 256, 0, stream>>>(free_stack, S, owner);
 }
 

@@ -18,7 +18,17 @@ struct PushArgs {
   uint64_t chunk;
   uint64_t nchunks;
   uint32_t worker;
+  float* span_head;       // pieces per block span (groups x chunk rows): nspans x D floats
+  float* span_tail;
+  uint32_t* long_list;    // nspans / 8 + 1 entries of scratch
+  uint32_t* long_count;   // one word, zeroed by the caller
 };
+
+// Number of block spans of a push of n rows with chunk length `chunk`.
+uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk);
+
+// Rows per push chunk for value length D and a batch of n rows.
+uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms);
 
 // One stored intent list (sorted unique keys, device count) and the sign of
 // its refcount event: +1 when its window opens, -1 when it closes.
