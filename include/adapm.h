@@ -111,6 +111,26 @@ adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
 adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                         const float* deltas);
 
+/* adapm_push without allocation.  The paper has no counterpart: this entry
+ * exists for callers that cannot let the library allocate device memory
+ * during a call -- a framework whose own allocator owns the memory budget,
+ * or a latency-critical loop in which cudaMalloc/cudaFree may synchronise
+ * the device.  Same result as adapm_push (same kernels and summation
+ * order), but its scratch is one file-scope device array of 16 MiB that
+ * every GPU which loads the library holds until the process exits.
+ *   - keys and deltas must be device arrays (ADAPM_EINVAL otherwise).
+ *   - A push whose sort and partial-sum buffers exceed the 16 MiB returns
+ *     ADAPM_EINVAL with the sizes in adapm_last_error().  Every n up to
+ *     about 500k rows fits at value_len 64, 69k at 200, 47k at 300, 28k at
+ *     512 and 14k at 1024.
+ *   - The first call on a device looks up the array's device address with
+ *     cudaGetSymbolAddress; make that first call before any stream capture.
+ *   - Every call (all contexts of the process) shares the one array: calls
+ *     that overlap on the GPU (different streams, different contexts) race.
+ *   - It allocates nothing: no cudaMalloc, cudaFree or pool allocation. */
+adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
+                                const float* deltas);
+
 /* Replica synchronisation (App. B.1.2): for every key with replicas,
  * main += the pending updates of all holders (ascending worker order), then
  * every holder's replica := main and its pending updates := 0. */

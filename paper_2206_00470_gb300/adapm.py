@@ -26,7 +26,7 @@ EXPORTS = [
     "adapm_push", "adapm_sync", "adapm_wait", "adapm_mf_step", "adapm_complex_step",
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
     "adapm_refcounts", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
-    "adapm_profile_read", "adapm_kernel_launches", "adapm_last_error",
+    "adapm_profile_read", "adapm_kernel_launches", "adapm_push_noalloc", "adapm_last_error",
 ]
 
 
@@ -96,6 +96,7 @@ def load(path=LIB_PATH):
         "adapm_profile_enable": [P, I],
         "adapm_profile_read": [P, P, P],
         "adapm_kernel_launches": [ctypes.POINTER(U64)],
+        "adapm_push_noalloc": [P, U32, P, U64, P],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -236,6 +237,14 @@ class ParameterManager:
         if d.n != k.n * self.D:
             raise ValueError("deltas must hold len(keys) * value_len floats")
         self._check(self._lib.adapm_push(self._h, worker, k.ptr, k.n, d.ptr))
+
+    def push_noalloc(self, worker, keys, deltas):
+        """adapm_push_noalloc: device tensors only; no allocation by the library."""
+        k = _keys(keys)
+        d = _floats(deltas)
+        if d.n != k.n * self.D:
+            raise ValueError("deltas must hold len(keys) * value_len floats")
+        self._check(self._lib.adapm_push_noalloc(self._h, worker, k.ptr, k.n, d.ptr))
 
     def sync(self):
         self._check(self._lib.adapm_sync(self._h))

@@ -268,6 +268,26 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
 
 }  // namespace
 
+bool adapm::ctx_view(adapm_ctx* ctx, CtxView* out) {
+  if (!ctx || !out) return false;
+  out->s = ctx->s;
+  out->dstate = ctx->dstate;
+  out->stream = ctx->stream;
+  out->device = ctx->device;
+  out->sms = ctx->sms;
+  out->bits = ctx->bits;
+  out->broken = ctx->broken;
+  return true;
+}
+
+void adapm::ctx_set_error(adapm_ctx* ctx, const char* msg) {
+  if (ctx) ctx->err = msg;
+}
+
+void adapm::ctx_add_push_rows(adapm_ctx* ctx, uint64_t n) {
+  if (ctx) ctx->push_rows_host += n;
+}
+
 extern "C" {
 
 adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {

@@ -15,6 +15,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+struct adapm_ctx;
+
 namespace adapm {
 
 constexpr uint32_t kNoKey = 0xFFFFFFFFu;          // sentinel: skipped element
@@ -94,5 +96,19 @@ int bits_for(uint64_t num_keys);   // bits covering [0, K] (K itself is the sent
 
 // Process-wide count of kernels launched by the library (capi.cu).
 void note_launches(uint64_t n);
+
+// What an entry point outside capi.cu needs of a context (capi.cu).
+struct CtxView {
+  Store s;
+  DevState* dstate;
+  cudaStream_t stream;
+  int device;
+  int sms;
+  int bits;
+  bool broken;
+};
+bool ctx_view(struct ::adapm_ctx* ctx, CtxView* out);
+void ctx_set_error(struct ::adapm_ctx* ctx, const char* msg);
+void ctx_add_push_rows(struct ::adapm_ctx* ctx, uint64_t n);
 
 }  // namespace adapm
