@@ -325,6 +325,9 @@ def sgns_batch(cfg, worker, clock, device="cpu"):
     """
     b = cfg.batch
     n_chunks = cfg.shard_len // b
+    if clock >= n_chunks:                       # this worker's shard is used up: idle
+        e = torch.empty(0, dtype=torch.int64, device=device)
+        return e, e.view(0, 2 * cfg.window), e.view(0, 2 * cfg.window, cfg.negatives)
     parts = []
     for ch in (clock - 1, clock, clock + 1):
         if 0 <= ch < n_chunks:
