@@ -34,7 +34,9 @@
  *     row for it is zero), ADAPM_ENOMEM when replica_capacity is exhausted
  *     (the replicas of that call are not created and reads of those keys go
  *     to the main copy), ADAPM_ESTATE for a refcount overflow (more than
- *     65535 overlapping intents of one worker on one key).
+ *     65535 overlapping intents of one worker on one key).  ADAPM_ETIMEOUT
+ *     is reserved for a bounded wait of one thread block on another that
+ *     gave up; no kernel of this version waits on another block.
  *   - ADAPM_ECUDA reports a CUDA runtime error; the context is then unusable.
  *   - No C++ exception crosses the ABI.  A context is driven by one host
  *     thread at a time.
@@ -121,7 +123,7 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
  *   - keys and deltas must be device arrays (ADAPM_EINVAL otherwise).
  *   - A push whose sort and partial-sum buffers exceed the 16 MiB returns
  *     ADAPM_EINVAL with the sizes in adapm_last_error().  Every n up to
- *     about 500k rows fits at value_len 64, 69k at 200, 47k at 300, 28k at
+ *     about 470k rows fits at value_len 64, 69k at 200, 47k at 300, 28k at
  *     512 and 14k at 1024.
  *   - The first call on a device looks up the array's device address with
  *     cudaGetSymbolAddress; make that first call before any stream capture.

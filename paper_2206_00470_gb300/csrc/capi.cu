@@ -231,10 +231,10 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &kb, n));
   CK(pool_alloc(ctx, &va, n));
   CK(pool_alloc(ctx, &vb, n));
-  CK(pool_alloc(ctx, &hist, sort_hist_words(n)));
+  CK(pool_alloc(ctx, &hist, sort_hist_words(n, ctx->bits)));
   launch_prep_keys(dkeys, n, ctx->s.K, ka, ctx->dstate, allow_nokey, ctx->sms, ctx->stream);
   uint32_t *sk = nullptr, *sp = nullptr;
-  radix_sort(ka, kb, va, vb, true, true, n, ctx->bits, hist, ctx->stream, &sk, &sp);
+  radix_sort(ka, kb, va, vb, true, true, n, ctx->bits, hist, ctx->dstate, ctx->stream, &sk, &sp);
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
   const uint64_t nspans = push_spans(ctx->s.D, n, chunk);
@@ -405,11 +405,12 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
     uint32_t *ka = nullptr, *kb = nullptr, *hist = nullptr, *tmp = nullptr;
     CK(pool_alloc(ctx, &ka, n));
     CK(pool_alloc(ctx, &kb, n));
-    CK(pool_alloc(ctx, &hist, sort_hist_words(n)));
+    CK(pool_alloc(ctx, &hist, sort_hist_words(n, ctx->bits)));
     CK(pool_alloc(ctx, &tmp, compact_tmp_words(n)));
     launch_prep_keys(in.dev, n, ctx->s.K, ka, ctx->dstate, false, ctx->sms, ctx->stream);
     uint32_t *sk = nullptr, *sv = nullptr;
-    radix_sort(ka, kb, nullptr, nullptr, false, false, n, ctx->bits, hist, ctx->stream, &sk, &sv);
+    radix_sort(ka, kb, nullptr, nullptr, false, false, n, ctx->bits, hist, ctx->dstate, ctx->stream,
+               &sk, &sv);
     unique_sorted(sk, n, L.keys, L.count, tmp, ctx->stream);
     pool_free(ctx, in.owned);
     pool_free(ctx, ka);
@@ -524,6 +525,7 @@ adapm_status adapm_wait(adapm_ctx* ctx) {
   if (errors & ERR_KEY_RANGE) return fail(ctx, ADAPM_ERANGE, "a key >= num_keys was passed");
   if (errors & ERR_NO_SLOTS) return fail(ctx, ADAPM_ENOMEM, "replica capacity exhausted");
   if (errors & ERR_REFCOUNT) return fail(ctx, ADAPM_ESTATE, "intent refcount overflow");
+  if (errors & ERR_TIMEOUT) return fail(ctx, ADAPM_ETIMEOUT, "a bounded device wait gave up");
   return ADAPM_OK;
 }
 

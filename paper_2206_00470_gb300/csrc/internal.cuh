@@ -28,6 +28,7 @@ enum ErrBits : uint32_t {
   ERR_KEY_RANGE = 1u,   // a key >= K was passed
   ERR_NO_SLOTS = 2u,    // replica capacity exhausted
   ERR_REFCOUNT = 4u,    // refcount over/underflow
+  ERR_TIMEOUT = 8u,     // a bounded wait on another block gave up
 };
 
 struct DevState {
@@ -72,15 +73,16 @@ __device__ __forceinline__ void set_error(DevState* st, uint32_t bits) {
 }
 
 // ---- radix sort / compaction (sort.cu) --------------------------------------
-// Sort n uint32 keys (with uint32 values if vals_in != nullptr or iota_vals)
-// by their low `bits` bits, stable, on `stream`.  Buffers a/b (keys) and
-// va/vb (values) are ping-pong space of n elements each; the result ends in
-// the buffer returned through *keys_out / *vals_out.  `hist` needs
-// sort_hist_words(n) uint32 words.
-size_t sort_hist_words(uint64_t n);
+// Sort n uint32 keys (with uint32 values if with_vals; iota_vals = the
+// values are the positions 0..n-1) by their low `bits` bits, stable, on
+// `stream`.  Buffers a/b (keys) and va/vb (values) are ping-pong space of n
+// elements each; the result ends in the buffer returned through *keys_out /
+// *vals_out.  `hist` is scratch of sort_hist_words(n, bits) uint32 words
+// (8-byte aligned); `st` receives ERR_TIMEOUT if a look-back wait gives up.
+size_t sort_hist_words(uint64_t n, int bits);
 void radix_sort(uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, bool with_vals,
-                bool iota_vals, uint64_t n, int bits, uint32_t* hist, cudaStream_t stream,
-                uint32_t** keys_out, uint32_t** vals_out);
+                bool iota_vals, uint64_t n, int bits, uint32_t* hist, DevState* st,
+                cudaStream_t stream, uint32_t** keys_out, uint32_t** vals_out);
 
 // Compact the distinct keys of a sorted array (dropping kNoKey) into out;
 // the count goes to *count (device).  tmp needs compact_tmp_words(n) words.
