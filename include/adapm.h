@@ -107,7 +107,8 @@ adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
 /* Write n delta rows: the rows of each distinct key are summed and the sum is
  * added to the worker's replica (its value and its pending-update
  * accumulator) or, without a replica, to the main copy (Sec. 4, App. B.1.2).
- * deltas: n*D floats, row i for keys[i].  Summation: rows in order of
+ * deltas: n*D floats, row i for keys[i] (a device array that is not 16-byte
+ * aligned is first copied to an aligned buffer).  Summation: rows in order of
  * appearance within fixed chunks of the key-sorted batch, chunk sums in
  * chunk order; deterministic for a given input. */
 adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
@@ -120,7 +121,8 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
  * the device.  Same result as adapm_push (same kernels and summation
  * order), but its scratch is one file-scope device array of 16 MiB that
  * every GPU which loads the library holds until the process exits.
- *   - keys and deltas must be device arrays (ADAPM_EINVAL otherwise).
+ *   - keys and deltas must be device arrays, deltas 16-byte aligned
+ *     (ADAPM_EINVAL otherwise).
  *   - A push whose sort and partial-sum buffers exceed the 16 MiB returns
  *     ADAPM_EINVAL with the sizes in adapm_last_error().  Every n up to
  *     about 470k rows fits at value_len 64, 69k at 200, 47k at 300, 28k at

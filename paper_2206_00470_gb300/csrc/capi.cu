@@ -500,6 +500,16 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
   Input<float> id;
   CK(stage_in(ctx, keys, n, &ik));
   CK(stage_in(ctx, deltas, n * ctx->s.D, &id));
+  if (reinterpret_cast<uintptr_t>(id.dev) % 16 != 0) {
+    // the push copies whole rows with the bulk-copy engine: 16-byte aligned rows
+    float* aligned = nullptr;
+    CK(pool_alloc(ctx, &aligned, n * ctx->s.D));
+    CK(cudaMemcpyAsync(aligned, id.dev, n * ctx->s.D * sizeof(float), cudaMemcpyDeviceToDevice,
+                       ctx->stream));
+    pool_free(ctx, id.owned);
+    id.owned = aligned;
+    id.dev = aligned;
+  }
   st = push_device(ctx, worker, ik.dev, n, id.dev, false);
   pool_free(ctx, ik.owned);
   pool_free(ctx, id.owned);

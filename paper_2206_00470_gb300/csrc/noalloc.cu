@@ -116,6 +116,10 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
     ctx_set_error(ctx, "adapm_push_noalloc takes device arrays only");
     return ADAPM_EINVAL;
   }
+  if (reinterpret_cast<uintptr_t>(deltas) % 16 != 0) {
+    ctx_set_error(ctx, "adapm_push_noalloc needs 16-byte aligned delta rows");
+    return ADAPM_EINVAL;
+  }
   const Layout L = layout(v.s.D, n, v.sms);
   if (L.total > kScratchBytes) {
     char msg[160];

@@ -384,12 +384,18 @@ sgns_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ centres, cons
   block_loss(lsum, o.loss_part);
 }
 
-__global__ void loss_reduce_kernel(const double* part, unsigned nparts, double* out) {
-  if (threadIdx.x == 0 && blockIdx.x == 0) {
-    double t = 0.0;
-    for (unsigned i = 0; i < nparts; ++i) t += part[i];
-    *out = t;
+// one block: thread t sums partials t, t+256, ... in order, then a fixed tree
+__global__ void __launch_bounds__(kThreads) loss_reduce_kernel(const double* part, unsigned nparts, double* out) {
+  __shared__ double sm[kThreads];
+  double t = 0.0;
+  for (unsigned i = threadIdx.x; i < nparts; i += kThreads) t += part[i];
+  sm[threadIdx.x] = t;
+  __syncthreads();
+  for (int w = kThreads / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) sm[threadIdx.x] += sm[threadIdx.x + w];
+    __syncthreads();
   }
+  if (threadIdx.x == 0) *out = sm[0];
 }
 
 }  // namespace
@@ -437,7 +443,7 @@ void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const
 
 void launch_loss_reduce(const double* part, unsigned nparts, double* out, cudaStream_t stream) {
   note_launches(1);
-  loss_reduce_kernel<<<1, 32, 0, stream>>>(part, nparts, out);
+  loss_reduce_kernel<<<1, kThreads, 0, stream>>>(part, nparts, out);
 }
 
 }  // namespace adapm

@@ -161,12 +161,18 @@ constexpr int kPushSpan = 1024;
 constexpr int kShortSpan = 8;
 
 template <int G, int C, int R>
-__global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 3) push_chunks_kernel(Store s, PushArgs a) {
+__global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 4) push_chunks_kernel(Store s, PushArgs a) {
   constexpr int NG = kThreads / G;
   const uint32_t CH = (uint32_t)a.chunk;            // rows per group, NG * CH <= kPushSpan
   const uint32_t span = NG * CH;
   __shared__ uint32_t sk[kPushSpan + 2];   // sk[0]: key before the span; sk[1+len]: key after it
-  __shared__ uint32_t sp[kPushSpan];
+  __shared__ uint32_t sp[kPushSpan];       // source row of each sorted position
+  __shared__ int32_t ss[kPushSpan];        // target slot of rows that end a whole segment
+  __shared__ uint8_t sf[kPushSpan];        // row flags (below)
+  // flags: bit0 a piece ends at this row, bit1 that piece began inside the
+  // row's chunk, bit2 the key's segment ends here, bit3 a piece begins here,
+  // bit4 the row holds a key (not a skipped one); a row with bits 0-2 all set
+  // ends a segment that lies inside one chunk
   const int lane = threadIdx.x & (G - 1);
   const int gi = threadIdx.x / G;
   const uint32_t D4 = s.D >> 2;
@@ -190,88 +196,84 @@ __global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 3) push_chunks_kernel(S
       sk[1 + len] = P0 + len < a.n ? a.skeys[P0 + len] : kNoKey;
     }
     __syncthreads();
+    // per-row control, one thread per row, and the slot of every whole segment
+    for (uint32_t i = threadIdx.x; i < len; i += kThreads) {
+      const uint32_t k = sk[1 + i];
+      uint8_t f = 0;
+      int32_t slot = -2;
+      if (k != kNoKey) {
+        const uint32_t cs = i - i % CH;                          // first row of the chunk
+        const uint32_t ce = cs + CH < len ? cs + CH : len;        // end of the chunk
+        const bool seg_begin = (P0 + i == 0) || sk[i] != k;       // sk[i] is the key of row i-1
+        const bool seg_end = (P0 + i + 1 >= a.n) || sk[1 + i + 1] != k;
+        const bool started = (P0 + cs == 0) || sk[cs] != k;       // piece began inside the chunk
+        const bool piece_end = seg_end || i + 1 == ce;
+        f = (piece_end ? 1 : 0) | (started ? 2 : 0) | (seg_end ? 4 : 0) |
+            ((seg_begin || i == cs) ? 8 : 0) | 16;
+        if (seg_begin) ++heads;
+        if ((f & 7) == 7) slot = mapw[k];
+      }
+      sf[i] = f;
+      ss[i] = slot;
+    }
+    __syncthreads();
     const uint32_t p0 = gi * CH;
     const uint32_t p1 = p0 + CH < len ? p0 + CH : len;
     const uint64_t j = P0 / CH + gi;                 // global chunk index
-    const bool has_prev = P0 + p0 > 0;
-    uint32_t cur = 0;
-    bool cur_valid = false, cur_started = false;
     float4 run[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) run[c] = f4zero();
     for (uint32_t p = p0; p < p1; p += R) {
+      // one round of loads: delta rows and the targets of whole segments ending here
+      uint8_t f[R];
+      int32_t sl[R];
       uint32_t k[R];
-      float4 d[R][C];
+      float4 d[R][C], tv[R][C], ta[R][C];
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         const bool v = p + r < p1;
+        f[r] = v ? sf[p + r] : 0;
+        sl[r] = (f[r] & 7) == 7 ? ss[p + r] : -2;
         k[r] = v ? sk[1 + p + r] : kNoKey;
         const uint32_t src = v ? sp[p + r] : 0u;
+        const float4* tvp = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          d[r][c] = (v && k[r] != kNoKey && col < D4) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
+          const bool cv = col < D4;
+          d[r][c] = ((f[r] & 16) && cv) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
+          tv[r][c] = (sl[r] != -2 && cv) ? tvp[col] : f4zero();
+          ta[r][c] = (sl[r] >= 0 && cv) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
         }
       }
-      uint32_t fl[R];   // bit0 piece ends here, bit1 piece started in chunk, bit2 segment ends here
+      // running sums in position order, then the stores
 #pragma unroll
       for (int r = 0; r < R; ++r) {
-        fl[r] = 0;
-        if (p + r < p1) {
-          if (!cur_valid || k[r] != cur) {
-            cur = k[r];
-            cur_valid = true;
-            cur_started = (p + r > p0) || !has_prev || sk[p0] != k[r];
-            if (cur_started && k[r] != kNoKey) ++heads;
 #pragma unroll
-            for (int c = 0; c < C; ++c) run[c] = f4zero();
-          }
+        for (int c = 0; c < C; ++c) {
+          run[c] = (f[r] & 8) ? d[r][c] : f4add(run[c], d[r][c]);
+          d[r][c] = run[c];
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if (sl[r] != -2) {
+          float4* dst = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
 #pragma unroll
           for (int c = 0; c < C; ++c) {
-            run[c] = f4add(run[c], d[r][c]);
-            d[r][c] = run[c];
+            const uint32_t col = lane + c * G;
+            if (col < D4) dst[col] = f4add(tv[r][c], d[r][c]);
           }
-          const uint32_t nxt = p + r + 1;             // local position of the next row
-          const bool kn_valid = P0 + nxt < a.n;
-          const bool seg_end = !kn_valid || sk[1 + nxt] != k[r];
-          const bool last = nxt == p1;
-          fl[r] = ((seg_end || last) ? 1u : 0u) | (cur_started ? 2u : 0u) | (seg_end ? 4u : 0u);
-          if (k[r] == kNoKey) fl[r] = 0;
-        }
-      }
-      // whole segments inside the chunk: add straight into their target
-      int32_t sl[R];
+          if (sl[r] >= 0) {
 #pragma unroll
-      for (int r = 0; r < R; ++r) sl[r] = fl[r] == 7u ? mapw[k[r]] : -2;
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        if (col < D4) {
-          float4 t[R];
-#pragma unroll
-          for (int r = 0; r < R; ++r)
-            if (sl[r] != -2)
-              t[r] = sl[r] >= 0 ? val4[(uint64_t)sl[r] * D4 + col] : main4[(uint64_t)k[r] * D4 + col];
-#pragma unroll
-          for (int r = 0; r < R; ++r) {
-            if (sl[r] != -2) {
-              float4* dst = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
-              dst[col] = f4add(t[r], d[r][c]);
+            for (int c = 0; c < C; ++c) {
+              const uint32_t col = lane + c * G;
+              if (col < D4) acc4[(uint64_t)sl[r] * D4 + col] = f4add(ta[r][c], d[r][c]);
             }
           }
-#pragma unroll
-          for (int r = 0; r < R; ++r)
-            if (sl[r] >= 0) t[r] = acc4[(uint64_t)sl[r] * D4 + col];
-#pragma unroll
-          for (int r = 0; r < R; ++r)
-            if (sl[r] >= 0) acc4[(uint64_t)sl[r] * D4 + col] = f4add(t[r], d[r][c]);
-        }
-      }
-      // pieces of segments cut by a chunk boundary: partial sums
-#pragma unroll
-      for (int r = 0; r < R; ++r) {
-        if ((fl[r] & 1u) && fl[r] != 7u) {
-          float4* dst = (fl[r] & 2u) ? pt4 : ph4;
+        } else if (f[r] & 1) {
+          // a piece of a segment cut by a chunk boundary: partial sum
+          float4* dst = (f[r] & 2) ? pt4 : ph4;
 #pragma unroll
           for (int c = 0; c < C; ++c) {
             const uint32_t col = lane + c * G;
@@ -346,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 3) push_chunks_kernel(S
       }
     }
   }
-  if (lane == 0 && heads) {
+  if (heads) {
     atomicAdd(&s.st->last_unique, heads);
     atomicAdd(&s.st->push_unique, (unsigned long long)heads);
   }
@@ -820,7 +822,7 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
   if (a.n == 0) return;
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    constexpr int R = 4 / C > 0 ? 4 / C : 1;
+    constexpr int R = 2 / C > 0 ? 2 / C : 1;
     uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
     const uint64_t cap = (uint64_t)sms * 4;
     note_launches(3);
