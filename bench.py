@@ -40,7 +40,7 @@ import torch  # noqa: E402
 from synth import hashgen  # noqa: E402
 from synth import workloads as wl  # noqa: E402
 
-METRIC = "pulled+pushed keys/s"
+METRIC = "pulled+pushed keys/s and training samples/s on 1 GB300; % of HBM roofline"
 UNIT = "keys/s"
 
 
@@ -102,7 +102,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -239,13 +239,18 @@ class MF:
     """Matrix factorisation 10M x 1M, rank 100 + AdaGrad: fused MF step per worker per clock."""
 
     def __init__(self, args, device, cfg=None):
-        self.cfg = cfg or wl.MF
+        import dataclasses
+        if cfg is None:
+            cfg = dataclasses.replace(wl.MF, rows=args.mf_rows or wl.MF.rows, cols=args.mf_cols or wl.MF.cols,
+                                      batch=args.batch or wl.MF.batch)
+        self.cfg = cfg
         c = self.cfg
         self.device = device
         self.K, self.D, self.W = c.num_keys, c.value_len, c.workers
         self.lookahead, self.span = c.lookahead, c.span
         self.row = self.D * 4
-        self.capacity = min(self.W * 2 * (self.lookahead + 1) * 2 * c.batch, 80_000_000)
+        # live replicas per worker: the distinct keys of one batch (2 per cell at most)
+        self.capacity = min(self.W * self.K, self.W * 4 * c.batch, 80_000_000)
         self.samples_per_step = self.W * c.batch
 
     def config(self):
@@ -314,7 +319,183 @@ class MF:
         return h2d, d2h
 
 
-WORKLOADS = {"micro": Micro, "mf": MF}
+class TinyMF(MF):
+    """The tiny 1,000 x 500 rank-16 MF (plain SGD, W=4, batch 256): the parity configuration."""
+
+    def __init__(self, args, device):
+        super().__init__(args, device, cfg=wl.TINY_MF)
+        self.capacity = self.K * self.W
+
+    def init_store(self):
+        c = self.cfg
+        return hashgen.init_store_torch(self.K, self.D, c.rank, c.seed, c.init_std, self.device)
+
+    def prepare(self, clocks):
+        c = self.cfg
+        data = wl.tiny_mf_dataset(c)
+        self.data = {}
+        for cl in range(clocks + self.lookahead + 1):
+            for w in range(self.W):
+                r, co, v = wl.tiny_mf_batch(c, data, w, cl % wl.tiny_mf_clocks(c, data[3]))
+                self.data[(w, cl)] = (r.to(torch.int32).to(self.device), co.to(torch.int32).to(self.device),
+                                      v.to(self.device), torch.cat([r, co]).to(torch.int32).to(self.device))
+        self.loss = torch.zeros(self.W, dtype=torch.float64, device=self.device)
+
+
+class ComplEx:
+    """ComplEx KGE, 5M entities + 800 relations, 2x128 + AdaGrad, 100 negatives, batch 4,096."""
+
+    def __init__(self, args, device):
+        self.cfg = wl.COMPLEX
+        c = self.cfg
+        self.device = device
+        self.K, self.D, self.W = c.num_keys, c.value_len, c.workers
+        self.lookahead, self.span = c.lookahead, c.span
+        self.row = self.D * 4
+        per = c.batch * (3 + c.negatives)
+        self.capacity = min(self.W * self.K, self.W * 2 * per, 40_000_000)
+        self.samples_per_step = self.W * c.batch
+
+    def config(self):
+        c = self.cfg
+        return {"workload": c.name, "entities": c.entities, "relations": c.relations,
+                "complex_dim": c.half_dim, "adagrad": True, "negatives": c.negatives,
+                "workers": c.workers, "batch_per_worker": c.batch, "zipf_entities": c.zipf_entities,
+                "zipf_relations": c.zipf_relations, "lookahead": c.lookahead, "intent_span": c.span,
+                "lr": c.lr}
+
+    def init_store(self):
+        c = self.cfg
+        return hashgen.init_store_torch(self.K, self.D, c.theta_dim, c.seed, c.init_std, self.device,
+                                        chunk_rows=1 << 20)
+
+    def prepare(self, clocks):
+        c = self.cfg
+        self.data = {}
+        for cl in range(clocks + self.lookahead + 1):
+            for w in range(self.W):
+                h, r, t, n = (x.to(torch.int32) for x in wl.complex_batch(c, w, cl, self.device))
+                self.data[(w, cl)] = (h, r, t, n.reshape(-1), torch.cat([h, r, t, n.reshape(-1)]))
+        self.loss = torch.zeros(self.W, dtype=torch.float64, device=self.device)
+
+    def start(self, pm):
+        for w in range(self.W):
+            for j in range(self.lookahead):
+                pm.intent(w, self.data[(w, j)][4], j, j + self.span)
+
+    def step(self, pm, cl, data=None, loss=None):
+        c = self.cfg
+        data = data or self.data
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, data[(w, j)][4], j, j + self.span)
+            h, r, t, n, _ = data[(w, cl)]
+            pm.complex_step(w, h, r, t, n, c.negatives, c.theta_dim, c.lr, c.eps,
+                            loss_out=(self.loss[w:w + 1] if loss is None else loss))
+            pm.advance_clock(w)
+        pm.sync()
+
+    def keys_per_step(self):
+        return 2 * self.W * self.cfg.batch * (3 + self.cfg.negatives)
+
+    def step_alg_bytes(self):
+        c = self.cfg
+        rows = c.batch * (3 + c.negatives)
+        # keys in (4 B per row), every row read once and one delta row + key written per row
+        return self.W * rows * (2 * self.row + 8)
+
+    def prepare_host(self, clocks):
+        self.hdata = {(w, cc): tuple(x.cpu().pin_memory() for x in self.data[(w, cc)]) for cc in clocks
+                      for w in range(self.W) if (w, cc) in self.data}
+        self.hloss = torch.zeros(1, dtype=torch.float64, pin_memory=True)
+
+    def step_host(self, pm, cl):
+        self.step(pm, cl, data=self.hdata, loss=self.hloss)
+
+    def host_bytes_per_step(self):
+        c = self.cfg
+        rows = c.batch * (3 + c.negatives)
+        return self.W * rows * 4 * 2, self.W * 8      # step keys + intent keys; batch loss
+
+
+class SGNS:
+    """Skip-gram with negative sampling, 700K vocabulary, dim 300, window 5, 25 negatives, batch 8,192."""
+
+    def __init__(self, args, device):
+        self.cfg = wl.SGNS
+        c = self.cfg
+        self.device = device
+        self.K, self.D, self.W = c.num_keys, c.value_len, c.workers
+        self.lookahead, self.span = c.lookahead, c.span
+        self.row = self.D * 4
+        self.n_ctx = 2 * c.window
+        self.per = 1 + self.n_ctx * (1 + c.negatives)
+        self.capacity = min(self.W * self.K, 40_000_000)
+        self.samples_per_step = self.W * c.batch
+
+    def config(self):
+        c = self.cfg
+        return {"workload": c.name, "vocab": c.vocab, "dim": c.dim, "window": c.window,
+                "negatives": c.negatives, "workers": c.workers, "batch_centres_per_worker": c.batch,
+                "zipf_s": c.zipf_s, "lookahead": c.lookahead, "intent_span": c.span, "lr": c.lr}
+
+    def init_store(self):
+        c = self.cfg
+        return hashgen.init_store_torch(self.K, self.D, c.dim, c.seed, c.init_std, self.device,
+                                        chunk_rows=1 << 20)
+
+    def prepare(self, clocks):
+        c = self.cfg
+        V = c.vocab
+        self.data = {}
+        for cl in range(clocks + self.lookahead + 1):
+            for w in range(self.W):
+                cen, ctx, neg = wl.sgns_batch(c, w, cl, self.device)
+                pres = ctx != wl.MISSING
+                keys = torch.cat([cen, V + ctx[pres], V + neg[pres].reshape(-1)]).to(torch.int32)
+                ctx32 = torch.where(pres, ctx, torch.full_like(ctx, 0xFFFFFFFF)).to(torch.int32)
+                self.data[(w, cl)] = (cen.to(torch.int32), ctx32.reshape(-1), neg.reshape(-1).to(torch.int32),
+                                      keys)
+        self.loss = torch.zeros(self.W, dtype=torch.float64, device=self.device)
+
+    def start(self, pm):
+        for w in range(self.W):
+            for j in range(self.lookahead):
+                pm.intent(w, self.data[(w, j)][3], j, j + self.span)
+
+    def step(self, pm, cl, data=None, loss=None):
+        c = self.cfg
+        data = data or self.data
+        for w in range(self.W):
+            j = cl + self.lookahead
+            pm.intent(w, data[(w, j)][3], j, j + self.span)
+            cen, ctx, neg, _ = data[(w, cl)]
+            pm.sgns_step(w, cen, ctx, neg, self.n_ctx, c.negatives, c.vocab, c.dim, c.lr,
+                         loss_out=(self.loss[w:w + 1] if loss is None else loss))
+            pm.advance_clock(w)
+        pm.sync()
+
+    def keys_per_step(self):
+        return 2 * self.W * self.cfg.batch * self.per
+
+    def step_alg_bytes(self):
+        # per centre: its rows read once, one delta row + key written per row
+        return self.W * self.cfg.batch * self.per * (2 * self.row + 8)
+
+    def prepare_host(self, clocks):
+        self.hdata = {(w, cc): tuple(x.cpu().pin_memory() for x in self.data[(w, cc)]) for cc in clocks
+                      for w in range(self.W) if (w, cc) in self.data}
+        self.hloss = torch.zeros(1, dtype=torch.float64, pin_memory=True)
+
+    def step_host(self, pm, cl):
+        self.step(pm, cl, data=self.hdata, loss=self.hloss)
+
+    def host_bytes_per_step(self):
+        c = self.cfg
+        return self.W * c.batch * self.per * 4 * 2, self.W * 8
+
+
+WORKLOADS = {"micro": Micro, "mf": MF, "tiny_mf": TinyMF, "complex": ComplEx, "sgns": SGNS}
 
 
 # ---------------------------------------------------------------------------
@@ -379,7 +560,6 @@ def run_ours(args, ws, rank, local):
         wk.step(pm, cl)
     end_ev.record()
     torch.cuda.synchronize()
-    clk = clocks.stop()
     launches = adapm.kernel_launches() - l0
     barrier(ws)
     ms = start_ev.elapsed_time(end_ev)
@@ -396,6 +576,7 @@ def run_ours(args, ws, rank, local):
     pm.profile_enable(False)
     s1 = pm.stats()
     pm.wait()
+    clk = clocks.stop()          # sampled over the timed and the profiled pass
 
     # -- end to end through the C ABI with pinned host buffers -------------------
     e2e_ms = None
@@ -542,6 +723,89 @@ def oracle_sample(workload, budget_s, args):
         desc = (f"{done} clocks of {cfg.workers} workers x {cfg.batch} cells of the 10M x 1M rank-100 "
                 f"AdaGrad workload (store restricted to the {touched.size} touched keys)")
         return 4 * cells / el, cells / el, desc
+    if workload == "tiny_mf":
+        cfg = wl.TINY_MF
+        data = wl.tiny_mf_dataset(cfg)
+        nclk = wl.tiny_mf_clocks(cfg, data[3])
+        init = hashgen.init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
+        pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init)
+        bt = {(w, c): [x.numpy() for x in wl.tiny_mf_batch(cfg, data, w, c)]
+              for w in range(cfg.workers) for c in range(nclk + cfg.lookahead + 1)}
+
+        def work(w, cl):
+            a, b, v = bt[(w, cl)]
+            return osteps.mf_step(pm, w, a, b, v, cfg.rank, cfg.lr, cfg.adagrad)
+
+        keys_of = lambda w, cl: np.concatenate(bt[(w, cl)][:2])  # noqa: E731
+        odriver.start(pm, cfg.workers, cfg.lookahead, cfg.span, keys_of)
+        t = time.perf_counter()
+        done = 0
+        while done < nclk and time.perf_counter() - t < budget_s:
+            odriver.clock(pm, cfg.workers, cfg.lookahead, cfg.span, done, keys_of, work)
+            done += 1
+        el = time.perf_counter() - t
+        cells = sum(bt[(w, c)][0].size for w in range(cfg.workers) for c in range(done))
+        return 4 * cells / el, cells / el, f"{done} clocks of the tiny MF workload (all {cfg.workers} workers)"
+    if workload in ("complex", "sgns"):
+        base = wl.COMPLEX if workload == "complex" else wl.SGNS
+        cfg = dataclasses.replace(base, batch=32 if workload == "complex" else 16)
+        nclk = 12
+        batches = {}
+        for cl in range(nclk + cfg.lookahead + 1):
+            for w in range(cfg.workers):
+                if workload == "complex":
+                    batches[(w, cl)] = [x.numpy() for x in wl.complex_batch(cfg, w, cl)]
+                else:
+                    batches[(w, cl)] = [x.numpy() for x in wl.sgns_batch(cfg, w, cl)]
+
+        def keys_full(b):
+            if workload == "complex":
+                return np.concatenate([b[0], b[1], b[2], b[3].reshape(-1)])
+            pres = b[1] != wl.MISSING
+            return np.concatenate([b[0], cfg.vocab + b[1][pres], cfg.vocab + b[2][pres].reshape(-1)])
+
+        touched = np.unique(np.concatenate([keys_full(b) for b in batches.values()]))
+        theta = cfg.theta_dim if workload == "complex" else cfg.dim
+        init = hashgen.init_rows_np(touched, cfg.value_len, theta, cfg.seed, cfg.init_std)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+        rel = lambda x: np.searchsorted(touched, x)  # noqa: E731
+
+        if workload == "complex":
+            def work(w, cl):
+                h, r, t_, n = batches[(w, cl)]
+                return osteps.complex_step(pm, w, rel(h), rel(r), rel(t_), rel(n), theta, cfg.lr, cfg.eps)
+            per = 3 + cfg.negatives
+        else:
+            # the store is relabelled: a token's output row is found through its relabelled key
+            class Relabelled:
+                def __init__(self, inner):
+                    self.inner = inner
+
+                def pull(self, w, keys):
+                    return self.inner.pull(w, rel(np.asarray(keys)))
+
+                def push(self, w, keys, d):
+                    return self.inner.push(w, rel(np.asarray(keys)), d)
+
+            rpm = Relabelled(pm)
+
+            def work(w, cl):
+                cen, ctx, neg = batches[(w, cl)]
+                return osteps.sgns_step(rpm, w, cen, ctx, neg, cfg.vocab, cfg.lr)
+            per = 1 + 2 * cfg.window * (1 + cfg.negatives)
+
+        keys_of = lambda w, cl: rel(keys_full(batches[(w, cl)]))  # noqa: E731
+        odriver.start(pm, cfg.workers, cfg.lookahead, cfg.span, keys_of)
+        t = time.perf_counter()
+        done = 0
+        while done < nclk and time.perf_counter() - t < budget_s:
+            odriver.clock(pm, cfg.workers, cfg.lookahead, cfg.span, done, keys_of, work)
+            done += 1
+        el = time.perf_counter() - t
+        samples = done * cfg.workers * cfg.batch
+        desc = (f"{done} clocks of {cfg.workers} workers x {cfg.batch} samples of the {base.name} workload "
+                f"(store restricted to the {touched.size} touched keys)")
+        return 2 * samples * per / el, samples / el, desc
     raise ValueError(workload)
 
 
@@ -577,11 +841,13 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="micro", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="mf", choices=sorted(WORKLOADS))
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--zipf", type=float, default=None)
     ap.add_argument("--span", type=int, default=None)
     ap.add_argument("--keys", type=int, default=None, help="micro: key-space size (default 1e8)")
+    ap.add_argument("--mf-rows", type=int, default=None, help="mf: rows (default 10M)")
+    ap.add_argument("--mf-cols", type=int, default=None, help="mf: columns (default 1M)")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")

@@ -244,11 +244,13 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
   CK(pool_alloc(ctx, &bh, nspans * ctx->s.D));
   CK(pool_alloc(ctx, &bt, nspans * ctx->s.D));
-  CK(pool_alloc(ctx, &longs, nspans / 8 + 2));
+  float* lparts = nullptr;
+  CK(pool_alloc(ctx, &longs, push_long_list_words(nspans)));
+  CK(pool_alloc(ctx, &lparts, push_long_part_rows(nspans) * ctx->s.D));
   CK(cudaMemsetAsync(longs, 0, sizeof(uint32_t), ctx->stream));
   CK(cudaMemsetAsync(&ctx->dstate->last_unique, 0, sizeof(uint32_t), ctx->stream));
   ctx->push_rows_host += n;
-  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, bh, bt, longs + 1, longs};
+  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, bh, bt, longs + 1, longs, lparts};
   {
     ProfScope ps(ctx, 6);
     launch_push(ctx->s, a, ctx->sms, ctx->stream);
@@ -263,6 +265,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   pool_free(ctx, bh);
   pool_free(ctx, bt);
   pool_free(ctx, longs);
+  pool_free(ctx, lparts);
   return check_launch(ctx, "push");
 }
 

@@ -59,7 +59,7 @@ bool is_device_ptr(const void* p) {
 
 // Byte offsets of the scratch regions of one push of n rows.
 struct Layout {
-  size_t ka, kb, va, vb, hist, ph, pt, bh, bt, longs, total;
+  size_t ka, kb, va, vb, hist, ph, pt, bh, bt, longs, lparts, total;
   uint64_t chunk, nchunks, nspans;
 };
 
@@ -83,7 +83,8 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   L.pt = take(L.nchunks * D * 4);
   L.bh = take(L.nspans * D * 4);
   L.bt = take(L.nspans * D * 4);
-  L.longs = take((L.nspans / 8 + 2) * 4);
+  L.longs = take(adapm::push_long_list_words(L.nspans) * 4);
+  L.lparts = take(adapm::push_long_part_rows(L.nspans) * D * 4);
   L.total = off;
   return L;
 }
@@ -160,7 +161,8 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
              reinterpret_cast<float*>(base + L.bh),
              reinterpret_cast<float*>(base + L.bt),
              longs + 1,
-             longs};
+             longs,
+             reinterpret_cast<float*>(base + L.lparts)};
   launch_push(v.s, a, v.sms, v.stream);
   e = cudaGetLastError();
   if (e != cudaSuccess) {

@@ -3,6 +3,7 @@
 // main copy), computes loss and gradients in fp32 from those values, and
 // writes one delta row per row occurrence for the push that follows:
 //   AdaGrad rows [theta | a]:  delta = [-lr*g/sqrt(a + g*g + eps) | g*g]
+//   (1/sqrt evaluated with the correctly rounded __frsqrt_rn)
 //   plain SGD:                 delta = -lr*g
 // Losses: MF 1/2 (v - u.w)^2; ComplEx softplus(-y phi), phi = Re(sum h r
 // conj(t)) with rows [re | im]; SGNS softplus(-u_o.v_c) + sum softplus(u_n.v_c).
@@ -37,7 +38,7 @@ __device__ __forceinline__ float sigmoid_f(float x) {
 
 // AdaGrad delta of one float of gradient g with accumulator a
 __device__ __forceinline__ float ada_theta(float g, float a, float lr, float eps) {
-  return -lr * g / sqrtf(a + g * g + eps);
+  return -lr * g * __frsqrt_rn(a + g * g + eps);   // correctly rounded 1/sqrt
 }
 __device__ __forceinline__ float4 ada_theta4(float4 g, float4 a, float lr, float eps) {
   return make_float4(ada_theta(g.x, a.x, lr, eps), ada_theta(g.y, a.y, lr, eps),

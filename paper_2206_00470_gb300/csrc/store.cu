@@ -386,7 +386,18 @@ __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs 
     for (int t = 0; t < kShortSpan; ++t)
       if (span == t && cont[t]) ++span;
     if (span == kShortSpan) {
-      if (lane == 0) long_list[atomicAdd(long_count, 1u)] = (uint32_t)j;
+      if (lane == 0) {
+        // last piece m whose first position still holds kl (a monotone predicate)
+        uint64_t lo = j + 1 + kShortSpan, hi = a.nchunks - 1;
+        while (lo < hi) {
+          const uint64_t mid = (lo + hi + 1) / 2;
+          if (a.skeys[mid * CH] == kl) lo = mid; else hi = mid - 1;
+        }
+        const uint32_t e = atomicAdd(long_count, 1u);
+        long_list[4 * e] = (uint32_t)j;
+        long_list[4 * e + 1] = (uint32_t)lo;
+        long_list[4 * e + 2] = 0;             // finished work items of this entry
+      }
       continue;
     }
     float4 tot[C];
@@ -415,66 +426,90 @@ __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs 
   }
 }
 
-// One block per long segment: its groups sum strided subsets of the head
-// pieces in increasing chunk order, then group 0 adds the tail piece and the
-// group sums in group order (a fixed summation tree: deterministic).
+// Hot keys: a segment whose pieces run over more than kShortSpan further
+// spans.  Its head pieces j+1 .. m_end are cut into work items of kLongSub
+// pieces, spread over all blocks; a block sums its item (groups take strided
+// pieces in increasing order, then the group sums in group order) into
+// long_parts.  The block that finishes an entry's last item adds the tail
+// piece and the item sums in item order and applies the total.  Every sum has
+// a fixed order, so the result does not depend on which block finishes last.
+constexpr uint32_t kLongSub = 32;
+
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a, const uint32_t* long_list,
+__global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a, uint32_t* long_list,
                                                              const uint32_t* long_count) {
   constexpr int NG = kThreads / G;
   const uint64_t CH = a.chunk;
   __shared__ float4 part[NG][G * C];
-  __shared__ uint64_t s_mend;
+  __shared__ int s_last;
   const int lane = threadIdx.x & (G - 1);
   const int gi = threadIdx.x / G;
   const uint32_t D4 = s.D >> 2;
   const float4* ph4 = reinterpret_cast<const float4*>(a.part_head);
   const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
+  float4* lp4 = reinterpret_cast<float4*>(a.long_parts);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   const uint32_t nl = *long_count;
-  for (uint32_t e = blockIdx.x; e < nl; e += gridDim.x) {
-    const uint64_t j = long_list[e];
-    const uint32_t kl = a.skeys[(j + 1) * CH - 1];
-    if (threadIdx.x == 0) {
-      // last chunk m whose first position still holds kl (monotone predicate)
-      uint64_t lo = j + 1, hi = a.nchunks - 1;
-      while (lo < hi) {
-        const uint64_t mid = (lo + hi + 1) / 2;
-        if (a.skeys[mid * CH] == kl) lo = mid; else hi = mid - 1;
+  for (uint64_t q = blockIdx.x;; q += gridDim.x) {
+    // locate work item q: entry e, item it, first item of the entry `base`
+    uint64_t base = 0, it = 0, ns = 0, j = 0, m_end = 0;
+    uint32_t e = 0;
+    for (; e < nl; ++e) {
+      j = long_list[4 * e];
+      m_end = long_list[4 * e + 1];
+      ns = (m_end - j + kLongSub - 1) / kLongSub;
+      if (q < base + ns) {
+        it = q - base;
+        break;
       }
-      s_mend = lo;
+      base += ns;
     }
-    __syncthreads();
-    const uint64_t m_end = s_mend;
+    if (e == nl) break;
+    const uint64_t lo = j + 1 + it * kLongSub;
+    const uint64_t hi = lo + kLongSub - 1 < m_end ? lo + kLongSub - 1 : m_end;
     float4 acc[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) acc[c] = f4zero();
-    constexpr int U = 4 / C > 0 ? 4 / C : 1;
-    for (uint64_t m = j + 1 + gi; m <= m_end; m += (uint64_t)NG * U) {
-      float4 t[U][C];
+    constexpr int U = (kLongSub + NG - 1) / NG;
+    float4 t[U][C];
 #pragma unroll
-      for (int u = 0; u < U; ++u)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-        for (int c = 0; c < C; ++c) {
-          const uint32_t col = lane + c * G;
-          const uint64_t mm = m + (uint64_t)u * NG;
-          t[u][c] = (mm <= m_end && col < D4) ? ph4[mm * D4 + col] : f4zero();
-        }
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        const uint64_t m = lo + gi + (uint64_t)u * NG;
+        t[u][c] = (m <= hi && col < D4) ? ph4[m * D4 + col] : f4zero();
+      }
 #pragma unroll
-      for (int u = 0; u < U; ++u)
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-        for (int c = 0; c < C; ++c) acc[c] = f4add(acc[c], t[u][c]);
-    }
+      for (int c = 0; c < C; ++c) acc[c] = f4add(acc[c], t[u][c]);
 #pragma unroll
     for (int c = 0; c < C; ++c) part[gi][lane + c * G] = acc[c];
     __syncthreads();
     if (gi == 0) {
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        float4 tot = f4zero();
+        for (int g2 = 0; g2 < NG; ++g2) tot = f4add(tot, part[g2][lane + c * G]);
+        if (col < D4) lp4[q * D4 + col] = tot;
+      }
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(long_list + 4 * e + 2, 1u) == (uint32_t)(ns - 1);
+    __syncthreads();
+    if (s_last && gi == 0) {
+      __threadfence();
+      const uint32_t kl = a.skeys[(j + 1) * CH - 1];
       float4 tot[C];
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
         tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
-        for (int q = 0; q < NG; ++q) tot[c] = f4add(tot[c], part[q][lane + c * G]);
+        for (uint64_t i2 = 0; i2 < ns; ++i2)
+          if (col < D4) tot[c] = f4add(tot[c], __ldcg(lp4 + (base + i2) * D4 + col));
       }
       apply_sum<C>(s, mapw, kl, tot, lane, G);
     }
@@ -809,6 +844,9 @@ uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms) {
   return ch;
 }
 
+uint64_t push_long_list_words(uint64_t nspans) { return 4 * (nspans / 8 + 2) + 1; }
+uint64_t push_long_part_rows(uint64_t nspans) { return nspans / kLongSub + nspans / 8 + 2; }
+
 uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk) {
   uint64_t span = 0;
   dispatch_gc(D / 4, [&](auto Gc, auto) {
@@ -834,7 +872,7 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
     sp.nchunks = spans;
     push_fixup_kernel<G, C><<<grid_for(sp.nchunks, G, sms), kThreads, 0, stream>>>(s, sp, a.long_list,
                                                                                   a.long_count);
-    push_long_kernel<G, C><<<(unsigned)sms, kThreads, 0, stream>>>(s, sp, a.long_list, a.long_count);
+    push_long_kernel<G, C><<<(unsigned)sms * 2, kThreads, 0, stream>>>(s, sp, a.long_list, a.long_count);
   });
 }
 
