@@ -664,7 +664,7 @@ __global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, c
 // sync
 // ---------------------------------------------------------------------------
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s) {
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint64_t hw = (uint64_t)s.st->high_water;
@@ -673,67 +673,113 @@ __global__ void __launch_bounds__(kThreads) sync_kernel(Store s) {
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   uint32_t nkeys = 0, nreps = 0;
-  for (uint64_t sl = g; sl < hw; sl += ng) {
-    const unsigned long long owner = s.slot_owner[sl];
-    if (owner == kEmptySlot) continue;
-    const uint32_t w = (uint32_t)(owner >> 32);
-    const uint32_t k = (uint32_t)owner;
-    const uint32_t mask = s.holders[k];
-    if ((uint32_t)(__ffs(mask) - 1) != w) continue;   // the lowest holder merges
-    if (lane == 0) {
-      nkeys += 1;
-      nreps += (uint32_t)__popc(mask);
-    }
-    float4 m[C];
+  // R slots per group at a time: owners, holder masks, then (for keys held
+  // by one worker only, the common case) main and pending rows, each as one
+  // round of independent loads
+  constexpr int R = 4 / C > 0 ? 4 / C : 1;
+  for (uint64_t b = g * R; b < hw; b += ng * R) {
+    unsigned long long own[R];
+    uint32_t mk[R];
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t col = lane + c * G;
-      m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
-    }
-    constexpr int Q = 8 / C > 0 ? 8 / C : 1;
-    uint32_t mm = mask;
-    while (mm) {
-      int32_t hs[Q];
+    for (int r = 0; r < R; ++r) own[r] = b + r < hw ? s.slot_owner[b + r] : kEmptySlot;
 #pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        hs[q] = -1;
-        if (mm) {
-          const uint32_t b = __ffs(mm) - 1;
-          mm &= mm - 1;
-          hs[q] = s.map[(uint64_t)b * s.K + k];
-        }
+    for (int r = 0; r < R; ++r) mk[r] = own[r] != kEmptySlot ? s.holders[(uint32_t)own[r]] : 0u;
+    bool single[R];
+    float4 mv[R][C], av[R][C];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const uint32_t w = (uint32_t)(own[r] >> 32);
+      single[r] = own[r] != kEmptySlot && mk[r] == (1u << w);
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        const bool cv = single[r] && col < D4;
+        mv[r][c] = cv ? main4[(uint64_t)(uint32_t)own[r] * D4 + col] : f4zero();
+        av[r][c] = cv ? acc4[(b + r) * D4 + col] : f4zero();
       }
-      float4 t[Q][C];
-#pragma unroll
-      for (int q = 0; q < Q; ++q)
-#pragma unroll
-        for (int c = 0; c < C; ++c) {
-          const uint32_t col = lane + c * G;
-          t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
-        }
-#pragma unroll
-      for (int q = 0; q < Q; ++q)
-        if (hs[q] >= 0)
-#pragma unroll
-          for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
     }
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t col = lane + c * G;
-      if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
-    }
-    mm = mask;
-    while (mm) {
-      const uint32_t b = __ffs(mm) - 1;
-      mm &= mm - 1;
-      const int32_t h = s.map[(uint64_t)b * s.K + k];
-      if (h < 0) continue;
+    for (int r = 0; r < R; ++r) {
+      if (!single[r]) continue;
+      if (lane == 0) {
+        nkeys += 1;
+        nreps += 1;
+      }
+      const uint32_t k = (uint32_t)own[r];
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
         if (col < D4) {
-          val4[(uint64_t)h * D4 + col] = m[c];
-          acc4[(uint64_t)h * D4 + col] = f4zero();
+          const float4 m = f4add(mv[r][c], av[r][c]);
+          main4[(uint64_t)k * D4 + col] = m;
+          val4[(b + r) * D4 + col] = m;
+          acc4[(b + r) * D4 + col] = f4zero();
+        }
+      }
+    }
+    // keys with several holders: the lowest holder merges all of them
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (own[r] == kEmptySlot || single[r]) continue;
+      const uint32_t w = (uint32_t)(own[r] >> 32);
+      const uint32_t k = (uint32_t)own[r];
+      const uint32_t mask = mk[r];
+      if ((uint32_t)(__ffs(mask) - 1) != w) continue;   // the lowest holder merges
+      if (lane == 0) {
+        nkeys += 1;
+        nreps += (uint32_t)__popc(mask);
+      }
+      float4 m[C];
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
+      }
+      constexpr int Q = 4 / C > 0 ? 4 / C : 1;
+      uint32_t mm = mask;
+      while (mm) {
+        int32_t hs[Q];
+#pragma unroll
+        for (int q = 0; q < Q; ++q) {
+          hs[q] = -1;
+          if (mm) {
+            const uint32_t wb = __ffs(mm) - 1;
+            mm &= mm - 1;
+            hs[q] = s.map[(uint64_t)wb * s.K + k];
+          }
+        }
+        float4 t[Q][C];
+#pragma unroll
+        for (int q = 0; q < Q; ++q)
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
+          }
+#pragma unroll
+        for (int q = 0; q < Q; ++q)
+          if (hs[q] >= 0)
+#pragma unroll
+            for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
+      }
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
+      }
+      mm = mask;
+      while (mm) {
+        const uint32_t wb = __ffs(mm) - 1;
+        mm &= mm - 1;
+        const int32_t h = s.map[(uint64_t)wb * s.K + k];
+        if (h < 0) continue;
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          if (col < D4) {
+            val4[(uint64_t)h * D4 + col] = m[c];
+            acc4[(uint64_t)h * D4 + col] = f4zero();
+          }
         }
       }
     }
@@ -914,7 +960,8 @@ void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stre
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     note_launches(1);
-    sync_kernel<G, C><<<grid_for(slot_bound, G, sms), kThreads, 0, stream>>>(s);
+    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // slots per group, as in sync_kernel
+    sync_kernel<G, C><<<grid_for((slot_bound + R - 1) / R, G, sms), kThreads, 0, stream>>>(s);
   });
 }
 
