@@ -35,8 +35,10 @@
  *     (the replicas of that call are not created and reads of those keys go
  *     to the main copy), ADAPM_ESTATE for a refcount overflow (more than
  *     65535 overlapping intents of one worker on one key).  ADAPM_ETIMEOUT
- *     is reserved for a bounded wait of one thread block on another that
- *     gave up; no kernel of this version waits on another block.
+ *     reports that a bounded device-side wait gave up: the sort of keys runs
+ *     as one cooperative launch whose blocks meet at grid barriers, and a
+ *     barrier wait is limited.  Work enqueued after such a failure does not
+ *     touch the store, and the context is unusable afterwards (destroy it).
  *   - ADAPM_ECUDA reports a CUDA runtime error; the context is then unusable.
  *   - No C++ exception crosses the ABI.  A context is driven by one host
  *     thread at a time.

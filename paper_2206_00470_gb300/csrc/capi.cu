@@ -58,6 +58,7 @@ struct adapm_ctx {
   int64_t next_list = 0;
   std::string err;
   bool broken = false;
+  unsigned long long bar_base = 0;   // dstate->bar_arrivals once the queued sorts have run
   uint64_t push_rows_host = 0;
   bool prof = false;
   std::vector<std::tuple<int, cudaEvent_t, cudaEvent_t>> pending;
@@ -231,10 +232,10 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &kb, n));
   CK(pool_alloc(ctx, &va, n));
   CK(pool_alloc(ctx, &vb, n));
-  CK(pool_alloc(ctx, &hist, sort_hist_words(n, ctx->bits)));
-  launch_prep_keys(dkeys, n, ctx->s.K, ka, ctx->dstate, allow_nokey, ctx->sms, ctx->stream);
+  CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
   uint32_t *sk = nullptr, *sp = nullptr;
-  radix_sort(ka, kb, va, vb, true, true, n, ctx->bits, hist, ctx->dstate, ctx->stream, &sk, &sp);
+  CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, nullptr, nullptr,
+               ctx->sms, ctx->dstate, &ctx->bar_base, ctx->stream, &sk, &sp));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
   const uint64_t nspans = push_spans(ctx->s.D, n, chunk);
@@ -280,6 +281,7 @@ bool adapm::ctx_view(adapm_ctx* ctx, CtxView* out) {
   out->sms = ctx->sms;
   out->bits = ctx->bits;
   out->broken = ctx->broken;
+  out->bar_base = &ctx->bar_base;
   return true;
 }
 
@@ -405,21 +407,16 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   } else {
     Input<uint32_t> in;
     CK(stage_in(ctx, keys, n, &in));
-    uint32_t *ka = nullptr, *kb = nullptr, *hist = nullptr, *tmp = nullptr;
+    uint32_t *ka = nullptr, *kb = nullptr, *hist = nullptr;
     CK(pool_alloc(ctx, &ka, n));
     CK(pool_alloc(ctx, &kb, n));
-    CK(pool_alloc(ctx, &hist, sort_hist_words(n, ctx->bits)));
-    CK(pool_alloc(ctx, &tmp, compact_tmp_words(n)));
-    launch_prep_keys(in.dev, n, ctx->s.K, ka, ctx->dstate, false, ctx->sms, ctx->stream);
-    uint32_t *sk = nullptr, *sv = nullptr;
-    radix_sort(ka, kb, nullptr, nullptr, false, false, n, ctx->bits, hist, ctx->dstate, ctx->stream,
-               &sk, &sv);
-    unique_sorted(sk, n, L.keys, L.count, tmp, ctx->stream);
+    CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
+    CK(sort_keys(in.dev, n, ctx->s.K, false, ctx->bits, ka, kb, nullptr, nullptr, hist, L.keys, L.count,
+                 ctx->sms, ctx->dstate, &ctx->bar_base, ctx->stream, nullptr, nullptr));
     pool_free(ctx, in.owned);
     pool_free(ctx, ka);
     pool_free(ctx, kb);
     pool_free(ctx, hist);
-    pool_free(ctx, tmp);
   }
   const int64_t id = ctx->next_list++;
   ctx->lists[id] = L;
@@ -535,10 +532,13 @@ adapm_status adapm_wait(adapm_ctx* ctx) {
   uint32_t errors = 0;
   CK(cudaMemcpy(&errors, &ctx->dstate->errors, sizeof errors, cudaMemcpyDeviceToHost));
   if (errors) CK(cudaMemset(&ctx->dstate->errors, 0, sizeof errors));
+  if (errors & ERR_TIMEOUT) {
+    ctx->broken = true;   // the grid-barrier state of the sort is unknown
+    return fail(ctx, ADAPM_ETIMEOUT, "a bounded device wait gave up");
+  }
   if (errors & ERR_KEY_RANGE) return fail(ctx, ADAPM_ERANGE, "a key >= num_keys was passed");
   if (errors & ERR_NO_SLOTS) return fail(ctx, ADAPM_ENOMEM, "replica capacity exhausted");
   if (errors & ERR_REFCOUNT) return fail(ctx, ADAPM_ESTATE, "intent refcount overflow");
-  if (errors & ERR_TIMEOUT) return fail(ctx, ADAPM_ETIMEOUT, "a bounded device wait gave up");
   return ADAPM_OK;
 }
 

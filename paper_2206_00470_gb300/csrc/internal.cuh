@@ -48,6 +48,9 @@ struct DevState {
   unsigned long long push_unique;     // distinct keys over all pushes (cumulative)
   unsigned long long sync_keys;       // keys merged by sync (cumulative)
   unsigned long long sync_replicas;   // replicas refreshed by sync (cumulative)
+  // grid barriers of the sort: blocks arrived, over the context's lifetime
+  // (a line of its own, away from the counters above)
+  alignas(128) unsigned long long bar_arrivals;
 };
 
 // Plain view of the device state passed to kernels by value.
@@ -72,23 +75,35 @@ __device__ __forceinline__ void set_error(DevState* st, uint32_t bits) {
   atomicOr(&st->errors, bits);
 }
 
-// ---- radix sort / compaction (sort.cu) --------------------------------------
-// Sort n uint32 keys (with uint32 values if with_vals; iota_vals = the
-// values are the positions 0..n-1) by their low `bits` bits, stable, on
-// `stream`.  Buffers a/b (keys) and va/vb (values) are ping-pong space of n
-// elements each; the result ends in the buffer returned through *keys_out /
-// *vals_out.  `hist` is scratch of sort_hist_words(n, bits) uint32 words
-// (8-byte aligned); `st` receives ERR_TIMEOUT if a look-back wait gives up.
-size_t sort_hist_words(uint64_t n, int bits);
-void radix_sort(uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, bool with_vals,
-                bool iota_vals, uint64_t n, int bits, uint32_t* hist, DevState* st,
-                cudaStream_t stream, uint32_t** keys_out, uint32_t** vals_out);
+// True once a sort has given up (ERR_TIMEOUT): its output is incomplete and
+// the kernels that consume sorted keys return without touching the store.
+__device__ __forceinline__ bool sort_failed(const DevState* st) {
+  return (*reinterpret_cast<const volatile uint32_t*>(&st->errors) & ERR_TIMEOUT) != 0u;
+}
 
-// Compact the distinct keys of a sorted array (dropping kNoKey) into out;
-// the count goes to *count (device).  tmp needs compact_tmp_words(n) words.
+// ---- radix sort / compaction (sort.cu) --------------------------------------
+// Stable sort of n uint32 keys by their low `bits` bits in one cooperative
+// launch on `stream`.  `raw` (n keys, not modified) is the first pass's
+// input; a key >= K is sorted as kNoKey (after every valid key) and sets
+// ERR_KEY_RANGE unless allow_nokey and it equals kNoKey.
+// ka/kb are ping-pong space of n keys; with va/vb non-null the positions
+// 0..n-1 travel with the keys.  The sorted keys (and positions) end in the
+// buffers returned through *keys_out / *pos_out.  If uniq_out is non-null,
+// the distinct keys other than kNoKey are written to it ascending and their
+// number to *uniq_count (0 if the sort gave up).  `scratch` holds
+// sort_scratch_words(n) uint32 words.  *bar_base is the host's copy of
+// st->bar_arrivals, advanced by the launch.  If a grid-barrier wait gives
+// up, the kernel sets ERR_TIMEOUT and returns; every kernel that consumes a
+// sort checks that bit first and does nothing while it is set.
+size_t sort_scratch_words(uint64_t n);
+cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
+                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch,
+                      uint32_t* uniq_out, uint32_t* uniq_count, int sms, DevState* st,
+                      unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
+                      uint32_t** pos_out);
+
+// Stream compaction (a count / scan / write pass), tmp of compact_tmp_words(n).
 size_t compact_tmp_words(uint64_t n);
-void unique_sorted(const uint32_t* sorted, uint64_t n, uint32_t* out, uint32_t* count,
-                   uint32_t* tmp, cudaStream_t stream);
 
 // Keys k < K with map_w[k] >= 0, ascending, into out; count to *count.
 void compact_replica_keys(const int32_t* map_w, uint64_t K, uint32_t* out, uint32_t* count,
@@ -108,6 +123,7 @@ struct CtxView {
   int sms;
   int bits;
   bool broken;
+  unsigned long long* bar_base;   // the context's copy of dstate->bar_arrivals
 };
 bool ctx_view(struct ::adapm_ctx* ctx, CtxView* out);
 void ctx_set_error(struct ::adapm_ctx* ctx, const char* msg);

@@ -78,7 +78,7 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   L.kb = take(n * 4);
   L.va = take(n * 4);
   L.vb = take(n * 4);
-  L.hist = take(adapm::sort_hist_words(n, 32) * 4);
+  L.hist = take(adapm::sort_scratch_words(n) * 4);
   L.ph = take(L.nchunks * D * 4);
   L.pt = take(L.nchunks * D * 4);
   L.bh = take(L.nspans * D * 4);
@@ -145,10 +145,13 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
     return ADAPM_ECUDA;
   }
   ctx_add_push_rows(ctx, n);
-  launch_prep_keys(keys, n, v.s.K, at(L.ka), v.dstate, false, v.sms, v.stream);
   uint32_t *sk = nullptr, *sp = nullptr;
-  radix_sort(at(L.ka), at(L.kb), at(L.va), at(L.vb), true, true, n, v.bits, at(L.hist), v.dstate,
-             v.stream, &sk, &sp);
+  e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist),
+                nullptr, nullptr, v.sms, v.dstate, v.bar_base, v.stream, &sk, &sp);
+  if (e != cudaSuccess) {
+    ctx_set_error(ctx, cudaGetErrorString(e));
+    return ADAPM_ECUDA;
+  }
   PushArgs a{sk,
              sp,
              n,

@@ -1,18 +1,34 @@
-// Stable LSD radix sort of uint32 keys (optionally with uint32 values) and
-// stream compaction, for the intent table (sort + unique of the keys of one
-// Intent call, Sec. 3) and for push (grouping a batch's delta rows by key).
+// Stable LSD radix sort of uint32 keys (optionally carrying their positions)
+// and stream compaction, for the intent table (sort + unique of the keys of
+// one Intent call, Sec. 3) and for push (grouping a batch's delta rows by
+// key).
 //
 // Only ceil(log2(K + 1)) key bits are sorted, in ceil(bits / 9) passes of at
-// most 9 bits (512 buckets): 27-bit keys (100M) take 3 passes.  One pass =
-//   hist    per tile of 1024 keys, digit counts (shared-memory atomics)
-//   scan    one block per digit: exclusive prefix of that digit's counts over
-//           the tiles (digit-major table), digit total
-//   scatter per tile: stable rank of each key among equal digits of the tile
-//           (a warp-level multi-split: one ballot per digit bit gives the
-//           lanes with the same digit; per-warp digit counters in shared
-//           memory order the warps), then position = digit base + earlier
-//           tiles' count + rank
-// No block waits on another, so the passes have no serial dependency chain.
+// most 9 bits (512 buckets): 27-bit keys (100M) take 3 passes.  The whole
+// sort is ONE cooperative launch of B blocks (all resident at once), block b
+// owning the contiguous chunk [b*n/B, (b+1)*n/B) of every pass.  The first
+// pass's digit counts of each chunk go to column b of a 512 x B table, then
+// every pass is
+//   1. scan    grid barrier; warp j scans row d = j of the table (the
+//              exclusive prefix of digit d over the chunks) and its total
+//   2. scatter grid barrier; digit bases = exclusive scan of the totals;
+//              the chunk is ranked in sub-tiles of 2048 keys (a warp-level
+//              multi-split: one ballot per digit bit gives the lanes with
+//              equal digits), reordered by digit in shared memory and
+//              written out in runs of equal digit (coalesced stores); each
+//              written key adds to the next pass's table, in the column of
+//              the chunk its position falls in (one atomic per distinct
+//              digit and chunk of a warp)
+// so a pass costs two grid barriers.  With one sub-tile per chunk
+// (n <= 2048 B) the first pass's ranks are kept in registers from the
+// count.  The optional unique pass (count the first key of every run,
+// barrier, block offsets, write) is one more phase of the same launch.
+//
+// The grid barrier is a monotonic arrival counter in DevState: the host
+// knows how many barriers each launch passes and hands the next launch its
+// starting value.  Its wait is bounded; a wait that gives up sets
+// ERR_TIMEOUT and the kernel returns, and since all later barriers need
+// every block, the whole launch stops within one bounded wait.
 #include "internal.cuh"
 
 namespace adapm {
@@ -20,16 +36,29 @@ namespace adapm {
 namespace {
 
 constexpr int kSortThreads = 256;
-constexpr int kSortItems = 8;                      // compaction: keys per thread
-constexpr int kTile = kSortThreads * kSortItems;
-constexpr int kRankItems = 4;                      // sort passes: keys per thread
-constexpr int kRankTile = kSortThreads * kRankItems;
 constexpr int kWarps = kSortThreads / 32;
+constexpr int kItems = 8;                          // keys per thread per sub-tile
+constexpr int kSub = kSortThreads * kItems;        // 2048 keys per sub-tile
+constexpr int kRadixBits = 9;
+constexpr int kDigits = 1 << kRadixBits;           // 512
+constexpr int kDPT = kDigits / kSortThreads;       // digits per thread (2)
+constexpr uint32_t kMaxSortBlocks = 4096;
+constexpr uint32_t kSpinLimit = 1u << 21;          // polls of one barrier wait
+constexpr int kScratchHead = 32;                   // words before the totals
+
+constexpr int kCompactItems = 8;                   // compaction: keys per thread
+constexpr int kTile = kSortThreads * kCompactItems;
 
 __device__ __forceinline__ uint32_t lanemask_lt() {
   uint32_t m;
   asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
   return m;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
 }
 
 // Lanes of the warp whose `valid` flag and low `nbits` digit bits equal this
@@ -75,9 +104,6 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* t
   return before + x - v;
 }
 
-constexpr int kRadixBits = 9;
-constexpr int kDigits = 1 << kRadixBits;          // 512
-
 struct PassPlan {
   int passes;
   int per;
@@ -91,142 +117,384 @@ PassPlan plan_for(int bits) {
   return p;
 }
 
-// hist[d * nt + tile] = number of keys of the tile with digit d
-__global__ void __launch_bounds__(kSortThreads)
-tile_hist_kernel(const uint32_t* __restrict__ keys, uint64_t n, int shift, uint32_t mask,
-                 uint32_t* __restrict__ hist, uint32_t nt) {
-  __shared__ uint32_t h[kDigits];
-  for (int i = threadIdx.x; i < kDigits; i += kSortThreads) h[i] = 0;
-  __syncthreads();
-  const uint64_t t0 = (uint64_t)blockIdx.x * kRankTile;
-  uint32_t k[kRankItems];
-#pragma unroll
-  for (int it = 0; it < kRankItems; ++it) {
-    const uint64_t i = t0 + (uint64_t)it * kSortThreads + threadIdx.x;
-    k[it] = i < n ? keys[i] : 0u;
-  }
-#pragma unroll
-  for (int it = 0; it < kRankItems; ++it) {
-    const uint64_t i = t0 + (uint64_t)it * kSortThreads + threadIdx.x;
-    if (i < n) atomicAdd(&h[(k[it] >> shift) & mask], 1u);
-  }
-  __syncthreads();
-  for (uint32_t d = threadIdx.x; d <= mask; d += kSortThreads) hist[(uint64_t)d * nt + blockIdx.x] = h[d];
+struct SortArgs {
+  const uint32_t* raw;
+  uint64_t n;
+  uint64_t K;
+  uint32_t* ka;
+  uint32_t* kb;
+  uint32_t* va;
+  uint32_t* vb;
+  uint32_t* table;        // kDigits x gridDim.x (digit-major)
+  uint32_t* totals;       // kDigits
+  uint32_t* uniq_out;
+  uint32_t* uniq_count;
+  DevState* st;
+  unsigned long long bar_base;   // st->bar_arrivals when the launch starts
+  int allow_nokey;
+  int passes;
+  int per;
+  int bits;
+};
+
+struct SortSmem {
+  uint32_t wcnt[kWarps][kDigits];   // per-warp digit counts, then warp offsets
+  uint32_t sk[kSub];                // sub-tile keys in digit order
+  uint32_t sv[kSub];                // their positions
+  uint32_t base[kDigits];           // output position of the chunk's next key per digit
+  uint32_t lofs[kDigits];           // first index of each digit in the reordered sub-tile
+  uint32_t cnt[kDigits];            // digit counts (chunk in step 1, sub-tile in step 3)
+  uint32_t scan[kWarps];
+  int abort;
+};
+
+__device__ __forceinline__ unsigned long long ld_acquire64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
 }
 
-// one block per digit: exclusive prefix over tiles in place, digit total
-__global__ void __launch_bounds__(kSortThreads)
-digit_scan_kernel(uint32_t* __restrict__ hist, uint32_t nt, uint32_t* __restrict__ totals) {
-  __shared__ uint32_t sm[kWarps];
-  uint32_t* row = hist + (uint64_t)blockIdx.x * nt;
-  uint32_t carry = 0;
-  for (uint32_t b0 = 0; b0 < nt; b0 += kSortThreads) {
-    const uint32_t idx = b0 + threadIdx.x;
-    const uint32_t v = idx < nt ? row[idx] : 0u;
-    uint32_t tot;
-    const uint32_t ex = block_exclusive_scan<kSortThreads>(v, &tot, sm);
-    if (idx < nt) row[idx] = carry + ex;
-    carry += tot;
-  }
-  if (threadIdx.x == 0) totals[blockIdx.x] = carry;
-}
-
-// stable scatter of one tile: position = digit base + earlier tiles' count + rank
-template <bool VALS, bool IOTA>
-__global__ void __launch_bounds__(kSortThreads)
-tile_scatter_kernel(const uint32_t* __restrict__ kin, const uint32_t* __restrict__ vin,
-                    uint32_t* __restrict__ kout, uint32_t* __restrict__ vout, uint64_t n, int shift,
-                    int nbits, const uint32_t* __restrict__ hist, uint32_t nt,
-                    const uint32_t* __restrict__ totals) {
-  __shared__ uint32_t wcnt[kWarps][kDigits];
-  __shared__ uint32_t base_s[kDigits];
-  __shared__ uint32_t sm[kWarps];
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  const uint32_t mask = (1u << nbits) - 1u;
-  const uint32_t nd = mask + 1;
-  constexpr int DPT = kDigits / kSortThreads;
-  for (int i = threadIdx.x; i < kWarps * kDigits; i += kSortThreads) (&wcnt[0][0])[i] = 0;
-  {
-    // digit bases: exclusive scan of the digit totals (blocked, DPT per thread)
-    uint32_t v[DPT], local = 0;
-#pragma unroll
-    for (int q = 0; q < DPT; ++q) {
-      const uint32_t d = threadIdx.x * DPT + q;
-      v[q] = d < nd ? totals[d] : 0u;
-      local += v[q];
-    }
-    uint32_t total;
-    uint32_t run = block_exclusive_scan<kSortThreads>(local, &total, sm);
-#pragma unroll
-    for (int q = 0; q < DPT; ++q) {
-      const uint32_t d = threadIdx.x * DPT + q;
-      if (d < nd) base_s[d] = run + hist[(uint64_t)d * nt + blockIdx.x];
-      run += v[q];
-    }
-  }
-  const uint64_t t0 = (uint64_t)blockIdx.x * kRankTile;
-  uint32_t key[kRankItems], val[kRankItems], rank[kRankItems];
-#pragma unroll
-  for (int it = 0; it < kRankItems; ++it) {
-    // warp w owns tile positions [w*128, (w+1)*128), item-major then lane
-    const uint64_t i = t0 + ((uint64_t)(warp * kRankItems + it) << 5) + lane;
-    const bool valid = i < n;
-    key[it] = valid ? kin[i] : 0u;
-    if (VALS) val[it] = IOTA ? (uint32_t)i : (valid ? vin[i] : 0u);
-  }
+// Grid barrier on a monotonic arrival counter: the k-th barrier of a launch
+// waits, bounded, until the counter reaches base + k * gridDim.x.  Arrival
+// is a release add, the wait an acquire load.  Block-wide: every thread
+// calls it.
+__device__ bool grid_barrier(const SortArgs& a, uint32_t& nbar, SortSmem& sm) {
   __syncthreads();
-  const uint32_t lt = lanemask_lt();
-#pragma unroll
-  for (int it = 0; it < kRankItems; ++it) {
-    const uint64_t i = t0 + ((uint64_t)(warp * kRankItems + it) << 5) + lane;
-    const bool valid = i < n;
-    const uint32_t d = (key[it] >> shift) & mask;
-    const uint32_t peers = digit_peers(d, valid, nbits);
-    const uint32_t prior = valid ? wcnt[warp][d] : 0u;
-    rank[it] = prior + __popc(peers & lt);
-    __syncwarp();
-    if (valid && lane == __ffs(peers) - 1) wcnt[warp][d] = prior + __popc(peers);
-    __syncwarp();
-  }
-  __syncthreads();
-#pragma unroll
-  for (int q = 0; q < DPT; ++q) {
-    const uint32_t d = threadIdx.x + q * kSortThreads;
-    if (d < nd) {
-      uint32_t run = 0;
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const uint32_t c = wcnt[w][d];
-        wcnt[w][d] = run;
-        run += c;
+  ++nbar;
+  if (threadIdx.x == 0) {
+    const unsigned long long target = a.bar_base + (unsigned long long)nbar * gridDim.x;
+    asm volatile("red.release.gpu.global.add.u64 [%0], 1;" ::"l"(&a.st->bar_arrivals) : "memory");
+    uint32_t it = 0;
+    while (ld_acquire64(&a.st->bar_arrivals) < target) {
+      if (++it > kSpinLimit) {
+        set_error(a.st, ERR_TIMEOUT);
+        sm.abort = 1;
+        break;
       }
     }
   }
   __syncthreads();
+  return sm.abort == 0;
+}
+
+// Load a sub-tile [s0, s1) (warp w owns positions s0 + [256w, 256w + 256),
+// item-major then lane) and rank every key among the equal digits before it:
+// afterwards sm.wcnt[w][d] = keys of digit d in warps < w, sm.cnt[d] = keys
+// of digit d in the sub-tile, rank[it] = earlier keys of the same digit in
+// the same warp.  `first`: keys come from the caller's array (mapped to
+// kNoKey when out of range, positions are the indices).
+template <bool POS>
+__device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin, const uint32_t* vin,
+                                          bool first, uint64_t s0, uint64_t s1, int shift, int nbits,
+                                          uint32_t (&key)[kItems], uint32_t (&val)[kItems],
+                                          uint32_t (&rank)[kItems], bool& bad, SortSmem& sm) {
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < kWarps * kDigits; i += kSortThreads) (&sm.wcnt[0][0])[i] = 0;
 #pragma unroll
-  for (int it = 0; it < kRankItems; ++it) {
-    const uint64_t i = t0 + ((uint64_t)(warp * kRankItems + it) << 5) + lane;
-    if (i < n) {
-      const uint32_t d = (key[it] >> shift) & mask;
-      const uint32_t pos = base_s[d] + wcnt[warp][d] + rank[it];
-      kout[pos] = key[it];
-      if (VALS) vout[pos] = val[it];
+  for (int it = 0; it < kItems; ++it) {
+    const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+    const bool valid = i < s1;
+    uint32_t k = 0;
+    if (valid) {
+      if (first) {
+        k = __ldg(kin + i);
+        if (k >= a.K) {
+          if (!(a.allow_nokey && k == kNoKey)) bad = true;
+          k = kNoKey;
+        }
+      } else {
+        k = __ldcg(kin + i);
+      }
     }
+    key[it] = k;
+    if (POS) val[it] = first ? (uint32_t)i : (valid ? __ldcg(vin + i) : 0u);
   }
+  __syncthreads();
+  const uint32_t mask = (1u << nbits) - 1u;
+  const uint32_t lt = lanemask_lt();
+#pragma unroll
+  for (int it = 0; it < kItems; ++it) {
+    const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+    const bool valid = i < s1;
+    const uint32_t d = (key[it] >> shift) & mask;
+    const uint32_t peers = digit_peers(d, valid, nbits);
+    const uint32_t prior = valid ? sm.wcnt[warp][d] : 0u;
+    rank[it] = prior + __popc(peers & lt);
+    __syncwarp();
+    if (valid && lane == __ffs(peers) - 1) sm.wcnt[warp][d] = prior + __popc(peers);
+    __syncwarp();
+  }
+  __syncthreads();
+#pragma unroll
+  for (int q = 0; q < kDPT; ++q) {
+    const int d = threadIdx.x * kDPT + q;
+    uint32_t run = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const uint32_t c = sm.wcnt[w][d];
+      sm.wcnt[w][d] = run;
+      run += c;
+    }
+    sm.cnt[d] = run;
+  }
+  __syncthreads();
+}
+
+// Distinct keys (kNoKey dropped) of the sorted keys in [i, i + kCompactItems)
+// per thread, as flags.
+__device__ __forceinline__ uint32_t first_of_run_flags(const uint32_t* keys, uint64_t i0, uint64_t end,
+                                                       bool (&f)[kCompactItems]) {
+  uint32_t c = 0;
+  uint32_t prev = i0 > 0 && i0 < end ? __ldcg(keys + i0 - 1) : kNoKey;
+#pragma unroll
+  for (int j = 0; j < kCompactItems; ++j) {
+    const uint64_t i = i0 + j;
+    const uint32_t k = i < end ? __ldcg(keys + i) : kNoKey;
+    f[j] = i < end && k != kNoKey && (i == 0 || k != prev);
+    prev = k;
+    c += f[j] ? 1u : 0u;
+  }
+  return c;
+}
+
+// Number of grid barriers one sort_kernel launch passes.
+__host__ __device__ constexpr uint32_t sort_barriers(int passes, bool uniq) {
+  return 2u * (uint32_t)passes + (uniq ? 2u : 0u);
+}
+
+template <bool POS, bool UNIQ>
+__global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
+  __shared__ SortSmem sm;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const uint32_t B = gridDim.x;
+  const uint32_t b = blockIdx.x;
+  if (UNIQ && b == 0 && threadIdx.x == 0) *a.uniq_count = 0;
+  // an earlier sort gave up: the barrier state is unknown, so do nothing
+  if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
+  __syncthreads();
+  if (sm.abort) return;
+  uint32_t nbar = 0;
+  const uint64_t chunk = (a.n + B - 1) / B;
+  const uint64_t c0 = a.n < b * chunk ? a.n : b * chunk;
+  const uint64_t c1 = a.n < c0 + chunk ? a.n : c0 + chunk;
+  const bool single = c1 - c0 <= (uint64_t)kSub;
+  uint32_t* const table0 = a.table;                       // passes 0, 2, ...
+  uint32_t* const table1 = a.table + (uint64_t)kDigits * B;   // passes 1, 3, ...
+  const uint32_t* kin = a.raw;
+  const uint32_t* vin = nullptr;
+  uint32_t* kout = a.ka;
+  uint32_t* vout = a.va;
+  uint32_t key[kItems], val[kItems], rank[kItems];
+  bool bad = false;
+  // 0. first pass digit counts of the chunk (ranks kept when one sub-tile)
+  {
+    const int nbits = a.per < a.bits ? a.per : a.bits;
+    const uint32_t mask = (1u << nbits) - 1u;
+    if (single) {
+      load_rank<POS>(a, kin, vin, true, c0, c1, 0, nbits, key, val, rank, bad, sm);
+    } else {
+      for (int d = threadIdx.x; d < kDigits; d += kSortThreads) sm.cnt[d] = 0;
+      __syncthreads();
+      for (uint64_t i = c0 + threadIdx.x; i < c1; i += kSortThreads) {
+        uint32_t k = __ldg(kin + i);
+        if (k >= a.K) {
+          if (!(a.allow_nokey && k == kNoKey)) bad = true;
+          k = kNoKey;
+        }
+        atomicAdd(&sm.cnt[k & mask], 1u);
+      }
+      __syncthreads();
+    }
+    for (uint32_t d = threadIdx.x; d <= mask; d += kSortThreads) table0[(uint64_t)d * B + b] = sm.cnt[d];
+    if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) set_error(a.st, ERR_KEY_RANGE);
+    if (!grid_barrier(a, nbar, sm)) return;
+  }
+  int shift = 0;
+  for (int p = 0; p < a.passes; ++p) {
+    const bool first = p == 0;
+    const bool more = p + 1 < a.passes;
+    const int nbits = a.per < a.bits - shift ? a.per : a.bits - shift;
+    const uint32_t mask = (1u << nbits) - 1u;
+    const int nshift = shift + nbits;   // next pass
+    const int nnbits = more ? (a.per < a.bits - nshift ? a.per : a.bits - nshift) : 0;
+    const uint32_t nmask = (1u << nnbits) - 1u;
+    uint32_t* tcur = (p & 1) ? table1 : table0;
+    uint32_t* tnext = (p & 1) ? table0 : table1;
+    // 1. exclusive prefix of each digit over the chunks, digit totals, and
+    // the digit's row of the next pass's table cleared.  Up to 16 chunks: one
+    // thread per digit (its row in one round of loads); more: one warp per
+    // digit, its row read in batches of 256 chunks, eight independent
+    // coalesced loads per lane
+    if (B <= 16) {
+      for (uint32_t d = b * kSortThreads + threadIdx.x; d < kDigits; d += B * kSortThreads) {
+        if (more && d <= nmask)
+          for (uint32_t j = 0; j < B; ++j) tnext[(uint64_t)d * B + j] = 0u;
+        if (d > mask) continue;
+        uint32_t* row = tcur + (uint64_t)d * B;
+        uint32_t v[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = (uint32_t)j < B ? __ldcg(row + j) : 0u;
+        uint32_t run = 0;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          if ((uint32_t)j < B) row[j] = run;
+          run += v[j];
+        }
+        a.totals[d] = run;
+      }
+    } else {
+      for (uint32_t d = b * kWarps + warp; d < kDigits; d += B * kWarps) {
+        if (more && d <= nmask)
+          for (uint32_t j = lane; j < B; j += 32) tnext[(uint64_t)d * B + j] = 0u;
+        if (d > mask) continue;
+        uint32_t* row = tcur + (uint64_t)d * B;
+        uint32_t carry = 0;
+        for (uint32_t j0 = 0; j0 < B; j0 += 256) {
+          uint32_t v[8];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const uint32_t j = j0 + q * 32 + lane;
+            v[q] = j < B ? __ldcg(row + j) : 0u;
+          }
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            uint32_t x = v[q];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+              const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+              if (lane >= o) x += y;
+            }
+            const uint32_t j = j0 + q * 32 + lane;
+            if (j < B) row[j] = carry + x - v[q];
+            carry += __shfl_sync(0xFFFFFFFFu, x, 31);
+          }
+        }
+        if (lane == 0) a.totals[d] = carry;
+      }
+    }
+    if (!grid_barrier(a, nbar, sm)) return;
+    // 2. scatter: digit bases, then the chunk's sub-tiles in order; each
+    // written key is counted for the next pass in the chunk it lands in
+    {
+      uint32_t v[kDPT], local = 0;
+#pragma unroll
+      for (int q = 0; q < kDPT; ++q) {
+        const uint32_t d = threadIdx.x * kDPT + q;
+        v[q] = d <= mask ? __ldcg(a.totals + d) : 0u;
+        local += v[q];
+      }
+      uint32_t total;
+      uint32_t run = block_exclusive_scan<kSortThreads>(local, &total, sm.scan);
+#pragma unroll
+      for (int q = 0; q < kDPT; ++q) {
+        const uint32_t d = threadIdx.x * kDPT + q;
+        sm.base[d] = run + (d <= mask ? __ldcg(tcur + (uint64_t)d * B + b) : 0u);
+        run += v[q];
+      }
+    }
+    for (uint64_t s0 = c0; s0 < c1; s0 += kSub) {
+      const uint64_t s1 = s0 + kSub < c1 ? s0 + kSub : c1;
+      if (!(single && first)) load_rank<POS>(a, kin, vin, first, s0, s1, shift, nbits, key, val, rank, bad, sm);
+      {
+        uint32_t local = 0;
+#pragma unroll
+        for (int q = 0; q < kDPT; ++q) local += sm.cnt[threadIdx.x * kDPT + q];
+        uint32_t total;
+        uint32_t run = block_exclusive_scan<kSortThreads>(local, &total, sm.scan);
+#pragma unroll
+        for (int q = 0; q < kDPT; ++q) {
+          const int d = threadIdx.x * kDPT + q;
+          sm.lofs[d] = run;
+          run += sm.cnt[d];
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int it = 0; it < kItems; ++it) {
+        const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+        if (i < s1) {
+          const uint32_t d = (key[it] >> shift) & mask;
+          const uint32_t lp = sm.lofs[d] + sm.wcnt[warp][d] + rank[it];
+          sm.sk[lp] = key[it];
+          if (POS) sm.sv[lp] = val[it];
+        }
+      }
+      __syncthreads();
+      const uint32_t m = (uint32_t)(s1 - s0);
+      for (uint32_t i0 = 0; i0 < m; i0 += kSortThreads) {   // block-uniform trip count
+        const uint32_t i = i0 + threadIdx.x;
+        uint32_t tag = 0xFFFFFFFFu;
+        if (i < m) {
+          const uint32_t k = sm.sk[i];
+          const uint32_t d = (k >> shift) & mask;
+          const uint32_t pos = sm.base[d] + (i - sm.lofs[d]);
+          kout[pos] = k;
+          if (POS) vout[pos] = sm.sv[i];
+          if (more) tag = (((k >> nshift) & nmask) << 12) | (uint32_t)(pos / chunk);
+        }
+        if (more) {
+          // one atomic per distinct (digit, chunk) of the warp
+          const uint32_t peers = __match_any_sync(0xFFFFFFFFu, tag);
+          if (tag != 0xFFFFFFFFu && lane == __ffs(peers) - 1)
+            atomicAdd(tnext + (uint64_t)(tag >> 12) * B + (tag & 0xFFFu), (uint32_t)__popc(peers));
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < kDPT; ++q) {
+        const int d = threadIdx.x * kDPT + q;
+        sm.base[d] += sm.cnt[d];
+      }
+      __syncthreads();
+    }
+    if (more || UNIQ) {
+      if (!grid_barrier(a, nbar, sm)) return;
+    }
+    kin = kout;
+    vin = vout;
+    kout = kout == a.ka ? a.kb : a.ka;
+    vout = vout == a.va ? a.vb : a.va;
+    shift = nshift;
+  }
+  if (!UNIQ) return;
+  // unique: count, barrier, block offset, write
+  uint32_t cnt = 0;
+  for (uint64_t s0 = c0; s0 < c1; s0 += kTile) {
+    bool f[kCompactItems];
+    const uint64_t s1 = s0 + kTile < c1 ? s0 + kTile : c1;
+    cnt += first_of_run_flags(kin, s0 + (uint64_t)threadIdx.x * kCompactItems, s1, f);
+  }
+  {
+    uint32_t total;
+    block_exclusive_scan<kSortThreads>(cnt, &total, sm.scan);
+    if (threadIdx.x == 0) a.table[b] = total;
+  }
+  if (!grid_barrier(a, nbar, sm)) return;
+  uint32_t before = 0;
+  for (uint32_t j = threadIdx.x; j < b; j += kSortThreads) before += __ldcg(a.table + j);
+  {
+    uint32_t total;
+    block_exclusive_scan<kSortThreads>(before, &total, sm.scan);
+    before = total;
+  }
+  for (uint64_t s0 = c0; s0 < c1; s0 += kTile) {
+    bool f[kCompactItems];
+    const uint64_t s1 = s0 + kTile < c1 ? s0 + kTile : c1;
+    const uint64_t i0 = s0 + (uint64_t)threadIdx.x * kCompactItems;
+    const uint32_t c = first_of_run_flags(kin, i0, s1, f);
+    uint32_t total;
+    uint32_t pos = before + block_exclusive_scan<kSortThreads>(c, &total, sm.scan);
+#pragma unroll
+    for (int j = 0; j < kCompactItems; ++j)
+      if (f[j]) a.uniq_out[pos++] = __ldcg(kin + i0 + j);
+    before += total;
+  }
+  if (b == B - 1 && threadIdx.x == 0) *a.uniq_count = before;
 }
 
 // ---- compaction ------------------------------------------------------------
-
-struct UniqueSel {
-  const uint32_t* s;
-  uint64_t n;
-  __device__ bool flag(uint64_t i) const {
-    const uint32_t k = s[i];
-    return k != kNoKey && (i == 0 || s[i - 1] != k);
-  }
-  __device__ uint32_t value(uint64_t i) const { return s[i]; }
-};
 
 struct MapSel {
   const int32_t* m;
@@ -238,10 +506,10 @@ struct MapSel {
 template <class Sel>
 __global__ void __launch_bounds__(kSortThreads) compact_count_kernel(Sel sel, uint32_t* tile_cnt) {
   __shared__ uint32_t sm[kWarps];
-  const uint64_t start = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kSortItems;
+  const uint64_t start = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kCompactItems;
   uint32_t c = 0;
 #pragma unroll
-  for (int j = 0; j < kSortItems; ++j) {
+  for (int j = 0; j < kCompactItems; ++j) {
     const uint64_t i = start + j;
     if (i < sel.n && sel.flag(i)) ++c;
   }
@@ -269,11 +537,11 @@ template <class Sel>
 __global__ void __launch_bounds__(kSortThreads)
 compact_write_kernel(Sel sel, const uint32_t* __restrict__ tile_off, uint32_t* __restrict__ out) {
   __shared__ uint32_t sm[kWarps];
-  const uint64_t start = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kSortItems;
-  bool f[kSortItems];
+  const uint64_t start = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kCompactItems;
+  bool f[kCompactItems];
   uint32_t c = 0;
 #pragma unroll
-  for (int j = 0; j < kSortItems; ++j) {
+  for (int j = 0; j < kCompactItems; ++j) {
     const uint64_t i = start + j;
     f[j] = i < sel.n && sel.flag(i);
     c += f[j] ? 1u : 0u;
@@ -281,7 +549,7 @@ compact_write_kernel(Sel sel, const uint32_t* __restrict__ tile_off, uint32_t* _
   uint32_t tot;
   uint32_t pos = tile_off[blockIdx.x] + block_exclusive_scan<kSortThreads>(c, &tot, sm);
 #pragma unroll
-  for (int j = 0; j < kSortItems; ++j) {
+  for (int j = 0; j < kCompactItems; ++j) {
     if (f[j]) out[pos++] = sel.value(start + j);
   }
 }
@@ -299,6 +567,39 @@ void compact(Sel sel, uint32_t* out, uint32_t* count, uint32_t* tmp, cudaStream_
   compact_write_kernel<Sel><<<nb, kSortThreads, 0, stream>>>(sel, tmp, out);
 }
 
+// Resident blocks per SM of one sort_kernel instance (its shared memory and
+// registers), looked up once.
+template <bool POS, bool UNIQ>
+int sort_blocks_per_sm() {
+  static const int occ = [] {
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS, UNIQ>, kSortThreads, 0) !=
+        cudaSuccess) {
+      cudaGetLastError();
+      o = 1;
+    }
+    return o < 1 ? 1 : o;
+  }();
+  return occ;
+}
+
+template <bool POS, bool UNIQ>
+cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cudaStream_t stream) {
+  const int occ = sort_blocks_per_sm<POS, UNIQ>();
+  uint64_t B = (a.n + kSub - 1) / kSub;
+  const uint64_t resident = (uint64_t)sms * (occ < 4 ? occ : 4);
+  if (B > resident) B = resident;
+  if (B > kMaxSortBlocks) B = kMaxSortBlocks;
+  if (B < 1) B = 1;
+  a.bar_base = *bar_base;
+  void* params[] = {&a};
+  note_launches(1);
+  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, UNIQ>, dim3((unsigned)B),
+                                                    dim3(kSortThreads), params, 0, stream);
+  if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes, UNIQ) * B;
+  return e;
+}
+
 }  // namespace
 
 int bits_for(uint64_t num_keys) {
@@ -307,56 +608,51 @@ int bits_for(uint64_t num_keys) {
   return b;
 }
 
-size_t sort_hist_words(uint64_t n, int bits) {
-  (void)bits;
-  const uint64_t nt = (n + kRankTile - 1) / kRankTile;
-  return (size_t)(kDigits * nt + kDigits);
+size_t sort_scratch_words(uint64_t n) {
+  uint64_t rows = (n + kSub - 1) / kSub;
+  if (rows > kMaxSortBlocks) rows = kMaxSortBlocks;
+  if (rows < 1) rows = 1;
+  return (size_t)(kScratchHead + kDigits + 2 * rows * kDigits);   // totals, two tables
 }
 
-void radix_sort(uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, bool with_vals,
-                bool iota_vals, uint64_t n, int bits, uint32_t* hist, DevState* st,
-                cudaStream_t stream, uint32_t** keys_out, uint32_t** vals_out) {
-  (void)st;
-  uint32_t *kin = ka, *kout = kb, *vin = va, *vout = vb;
-  if (n == 0) {
-    *keys_out = kin;
-    *vals_out = vin;
-    return;
-  }
-  const uint32_t nt = (uint32_t)((n + kRankTile - 1) / kRankTile);
-  uint32_t* totals = hist + (uint64_t)kDigits * nt;
+cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
+                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch,
+                      uint32_t* uniq_out, uint32_t* uniq_count, int sms, DevState* st,
+                      unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
+                      uint32_t** pos_out) {
   const PassPlan pl = plan_for(bits);
-  int shift = 0;
-  for (int p = 0; p < pl.passes; ++p) {
-    const int b = pl.per < bits - shift ? pl.per : bits - shift;
-    const uint32_t mask = (1u << b) - 1u;
-    note_launches(3);
-    tile_hist_kernel<<<nt, kSortThreads, 0, stream>>>(kin, n, shift, mask, hist, nt);
-    digit_scan_kernel<<<mask + 1, kSortThreads, 0, stream>>>(hist, nt, totals);
-    if (!with_vals) {
-      tile_scatter_kernel<false, false><<<nt, kSortThreads, 0, stream>>>(
-          kin, nullptr, kout, nullptr, n, shift, b, hist, nt, totals);
-    } else if (p == 0 && iota_vals) {
-      tile_scatter_kernel<true, true><<<nt, kSortThreads, 0, stream>>>(
-          kin, nullptr, kout, vout, n, shift, b, hist, nt, totals);
-    } else {
-      tile_scatter_kernel<true, false><<<nt, kSortThreads, 0, stream>>>(
-          kin, vin, kout, vout, n, shift, b, hist, nt, totals);
-    }
-    uint32_t* t = kin; kin = kout; kout = t;
-    t = vin; vin = vout; vout = t;
-    shift += b;
+  if (keys_out) *keys_out = pl.passes % 2 ? ka : kb;
+  if (pos_out) *pos_out = va ? (pl.passes % 2 ? va : vb) : nullptr;
+  if (n == 0) {
+    if (uniq_count) return cudaMemsetAsync(uniq_count, 0, sizeof(uint32_t), stream);
+    return cudaSuccess;
   }
-  *keys_out = kin;
-  *vals_out = vin;
+  SortArgs a;
+  a.raw = raw;
+  a.n = n;
+  a.K = K;
+  a.ka = ka;
+  a.kb = kb;
+  a.va = va;
+  a.vb = vb;
+  a.totals = scratch + kScratchHead;
+  a.table = scratch + kScratchHead + kDigits;
+  a.uniq_out = uniq_out;
+  a.uniq_count = uniq_count;
+  a.st = st;
+  a.allow_nokey = allow_nokey ? 1 : 0;
+  a.passes = pl.passes;
+  a.per = pl.per;
+  a.bits = bits;
+  const bool pos = va != nullptr;
+  const bool uniq = uniq_out != nullptr;
+  if (pos && uniq) return launch_sort<true, true>(a, bar_base, sms, stream);
+  if (pos) return launch_sort<true, false>(a, bar_base, sms, stream);
+  if (uniq) return launch_sort<false, true>(a, bar_base, sms, stream);
+  return launch_sort<false, false>(a, bar_base, sms, stream);
 }
 
 size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile + 1); }
-
-void unique_sorted(const uint32_t* sorted, uint64_t n, uint32_t* out, uint32_t* count,
-                   uint32_t* tmp, cudaStream_t stream) {
-  compact(UniqueSel{sorted, n}, out, count, tmp, stream);
-}
 
 void compact_replica_keys(const int32_t* map_w, uint64_t K, uint32_t* out, uint32_t* count,
                           uint32_t* tmp, cudaStream_t stream) {

@@ -43,24 +43,6 @@ __device__ __forceinline__ uint64_t group_count() {
 }
 
 // ---------------------------------------------------------------------------
-// key preparation: copy, range check, sentinel for bad keys
-// ---------------------------------------------------------------------------
-__global__ void prep_keys_kernel(const uint32_t* __restrict__ in, uint64_t n, uint64_t K,
-                                 uint32_t* __restrict__ out, DevState* st, int allow_nokey) {
-  bool bad = false;
-  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-       i += (uint64_t)gridDim.x * blockDim.x) {
-    uint32_t k = in[i];
-    if (k >= K) {
-      if (!(allow_nokey && k == kNoKey)) bad = true;
-      k = kNoKey;
-    }
-    out[i] = k;
-  }
-  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(st, ERR_KEY_RANGE);
-}
-
-// ---------------------------------------------------------------------------
 // pull (and main-only gather for inspection when w < 0)
 // ---------------------------------------------------------------------------
 template <int G, int C, int R>
@@ -162,6 +144,7 @@ constexpr int kShortSpan = 8;
 
 template <int G, int C, int R>
 __global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 4) push_chunks_kernel(Store s, PushArgs a) {
+  if (sort_failed(s.st)) return;
   constexpr int NG = kThreads / G;
   const uint32_t CH = (uint32_t)a.chunk;            // rows per group, NG * CH <= kPushSpan
   const uint32_t span = NG * CH;
@@ -361,6 +344,7 @@ __global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 4) push_chunks_kernel(S
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs a, uint32_t* long_list,
                                                               uint32_t* long_count) {
+  if (sort_failed(s.st)) return;
   const uint64_t CH = a.chunk;
   const int lane = threadIdx.x & (G - 1);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
@@ -438,6 +422,7 @@ constexpr uint32_t kLongSub = 32;
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a, uint32_t* long_list,
                                                              const uint32_t* long_count) {
+  if (sort_failed(s.st)) return;
   constexpr int NG = kThreads / G;
   const uint64_t CH = a.chunk;
   __shared__ float4 part[NG][G * C];
@@ -521,7 +506,8 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
 // intent events -> refcounts -> create / evict lists
 // ---------------------------------------------------------------------------
 __global__ void events_add_kernel(const uint32_t* __restrict__ keys, const uint32_t* __restrict__ count,
-                                  int sign, int32_t* __restrict__ ev_delta) {
+                                  int sign, int32_t* __restrict__ ev_delta, const DevState* st) {
+  if (sort_failed(st)) return;
   const uint32_t n = *count;
   for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
     atomicAdd(ev_delta + keys[i], sign);
@@ -544,41 +530,69 @@ __device__ __forceinline__ void warp_append(bool want, uint32_t value, uint32_t*
   if (want) list[base + __popc(m & lanemask_lt_())] = value;
 }
 
+// Net refcount change of every listed key (4 keys per thread per round, each
+// step a round of independent accesses), appended to the create list (0 ->
+// >0) or the evict list (>0 -> 0, if a replica exists).
 __global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys,
                                     const uint32_t* __restrict__ count, uint32_t* create_list,
                                     uint32_t* evict_list) {
+  if (sort_failed(s.st)) return;
+  constexpr int Q = 4;
   const uint32_t n = *count;
   uint16_t* rcw = s.rc + (uint64_t)w * s.K;
-  const uint32_t stride = gridDim.x * blockDim.x;
-  for (uint32_t b = blockIdx.x * blockDim.x; b < n; b += stride) {   // warp-uniform trip count
-    const uint32_t i = b + threadIdx.x;
-    bool create = false, evict = false;
-    uint32_t k = 0;
-    if (i < n) {
-      k = keys[i];
-      const int32_t d = atomicExch(s.ev_delta + k, 0);
-      if (d != 0) {
-        const int32_t old = rcw[k];
-        int32_t nw = old + d;
+  const int32_t* mapw = s.map + (uint64_t)w * s.K;
+  const uint32_t stride = gridDim.x * blockDim.x * Q;
+  for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // warp-uniform trip count
+    uint32_t k[Q];
+    int32_t d[Q], old[Q];
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      k[q] = i < n ? keys[i] : 0u;
+    }
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      d[q] = i < n ? atomicExch(s.ev_delta + k[q], 0) : 0;
+    }
+#pragma unroll
+    for (int q = 0; q < Q; ++q) old[q] = d[q] != 0 ? (int32_t)rcw[k[q]] : 0;
+    bool create[Q], evict[Q];
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      create[q] = false;
+      evict[q] = false;
+      if (d[q] != 0) {
+        int32_t nw = old[q] + d[q];
         if (nw < 0 || nw > 65535) {
           set_error(s.st, ERR_REFCOUNT);
           nw = nw < 0 ? 0 : 65535;
         }
-        rcw[k] = (uint16_t)nw;
-        create = old == 0 && nw > 0;
-        // a key whose replica was never created (capacity exhausted) has nothing to destroy
-        evict = old > 0 && nw == 0 && s.map[(uint64_t)w * s.K + k] >= 0;
+        rcw[k[q]] = (uint16_t)nw;
+        create[q] = old[q] == 0 && nw > 0;
+        evict[q] = old[q] > 0 && nw == 0;
       }
     }
-    warp_append(create, k, &s.st->n_create, create_list);
-    warp_append(evict, k, &s.st->n_evict, evict_list);
+    // a key whose replica was never created (capacity exhausted) has nothing to destroy
+#pragma unroll
+    for (int q = 0; q < Q; ++q)
+      if (evict[q]) evict[q] = mapw[k[q]] >= 0;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      warp_append(create[q], k[q], &s.st->n_create, create_list);
+      warp_append(evict[q], k[q], &s.st->n_evict, evict_list);
+    }
   }
 }
 
 // evict: main[k] += acc[slot]; the freed slot goes on the stack at
-// free_top + i (every listed key holds a replica), so no atomics are needed
+// free_top + i (every listed key holds a replica), so no atomics are needed.
+// R keys per row group at a time: list entries, slots, then the rows, each
+// as one round of independent loads.
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) evict_kernel(Store s, uint32_t w, const uint32_t* __restrict__ list) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s, uint32_t w,
+                                                                       const uint32_t* __restrict__ list) {
+  constexpr int R = 4 / C > 0 ? 4 / C : 1;
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint32_t n = s.st->n_evict;
@@ -587,19 +601,37 @@ __global__ void __launch_bounds__(kThreads) evict_kernel(Store s, uint32_t w, co
   float4* main4 = reinterpret_cast<float4*>(s.main);
   const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  for (uint64_t i = g; i < n; i += ng) {
-    const uint32_t k = list[i];
-    const int32_t sl = mapw[k];
+  for (uint64_t i0 = g * R; i0 < n; i0 += ng * R) {
+    uint32_t k[R];
+    int32_t sl[R];
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t col = lane + c * G;
-      if (col < D4) main4[(uint64_t)k * D4 + col] = f4add(main4[(uint64_t)k * D4 + col], acc4[(uint64_t)sl * D4 + col]);
-    }
-    if (lane == 0) {
-      mapw[k] = -1;
-      atomicAnd(s.holders + k, ~(1u << w));
-      s.slot_owner[sl] = kEmptySlot;
-      s.free_stack[top + (int32_t)i] = sl;
+    for (int r = 0; r < R; ++r) k[r] = i0 + r < n ? list[i0 + r] : 0u;
+#pragma unroll
+    for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? mapw[k[r]] : 0;
+    float4 m[R][C], ac[R][C];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        const bool v = i0 + r < n && col < D4;
+        m[r][c] = v ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
+        ac[r][c] = v ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
+      }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (i0 + r >= n) break;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) main4[(uint64_t)k[r] * D4 + col] = f4add(m[r][c], ac[r][c]);
+      }
+      if (lane == 0) {
+        mapw[k[r]] = -1;
+        atomicAnd(s.holders + k[r], ~(1u << w));
+        s.slot_owner[sl[r]] = kEmptySlot;
+        s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
+      }
     }
   }
 }
@@ -628,9 +660,12 @@ __global__ void alloc_kernel(DevState* st, int32_t S) {
   if (S - st->alloc_base > st->high_water) st->high_water = S - st->alloc_base;
 }
 
-// create: val = main[k], acc = 0, take a slot from the stack
+// create: val = main[k], acc = 0, take a slot from the stack (R keys per
+// row group at a time, as in evict_kernel)
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, const uint32_t* __restrict__ list) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store s, uint32_t w,
+                                                                        const uint32_t* __restrict__ list) {
+  constexpr int R = 4 / C > 0 ? 4 / C : 1;
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint32_t n = s.st->n_create_ok;
@@ -640,22 +675,40 @@ __global__ void __launch_bounds__(kThreads) create_kernel(Store s, uint32_t w, c
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  for (uint64_t i = g; i < n; i += ng) {
-    const uint32_t k = list[i];
-    // slots popped from the top of the stack: lowest free slots come first
-    const int32_t sl = s.free_stack[base + (int32_t)(n - 1 - i)];
+  for (uint64_t i0 = g * R; i0 < n; i0 += ng * R) {
+    uint32_t k[R];
+    int32_t sl[R];
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t col = lane + c * G;
-      if (col < D4) {
-        val4[(uint64_t)sl * D4 + col] = main4[(uint64_t)k * D4 + col];
-        acc4[(uint64_t)sl * D4 + col] = f4zero();
-      }
+    for (int r = 0; r < R; ++r) {
+      const bool v = i0 + r < n;
+      k[r] = v ? list[i0 + r] : 0u;
+      // slots popped from the top of the stack: lowest free slots come first
+      sl[r] = v ? s.free_stack[base + (int32_t)(n - 1 - (i0 + r))] : 0;
     }
-    if (lane == 0) {
-      mapw[k] = sl;
-      atomicOr(s.holders + k, 1u << w);
-      s.slot_owner[sl] = ((unsigned long long)w << 32) | k;
+    float4 m[R][C];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        m[r][c] = (i0 + r < n && col < D4) ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
+      }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (i0 + r >= n) break;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) {
+          val4[(uint64_t)sl[r] * D4 + col] = m[r][c];
+          acc4[(uint64_t)sl[r] * D4 + col] = f4zero();
+        }
+      }
+      if (lane == 0) {
+        mapw[k[r]] = sl[r];
+        atomicOr(s.holders + k[r], 1u << w);
+        s.slot_owner[sl[r]] = ((unsigned long long)w << 32) | k[r];
+      }
     }
   }
 }
@@ -843,6 +896,17 @@ void dispatch_gc(uint32_t D4, F&& f) {
   else f(std::integral_constant<int, 32>{}, std::integral_constant<int, 8>{});
 }
 
+// The push kernels give each lane two float4 of a row where the row allows
+// it, so every row's control work (flags, slots, addresses) is shared by
+// half as many lanes.
+template <class F>
+void dispatch_push_gc(uint32_t D4, F&& f) {
+  if (D4 <= 8) f(std::integral_constant<int, 4>{}, std::integral_constant<int, 2>{});
+  else if (D4 <= 16) f(std::integral_constant<int, 8>{}, std::integral_constant<int, 2>{});
+  else if (D4 <= 32) f(std::integral_constant<int, 16>{}, std::integral_constant<int, 2>{});
+  else dispatch_gc(D4, f);
+}
+
 unsigned grid_for(uint64_t groups, int G, int sms) {
   const uint64_t per_block = kThreads / G;
   uint64_t b = (groups + per_block - 1) / per_block;
@@ -857,15 +921,6 @@ unsigned grid_for(uint64_t groups, int G, int sms) {
 // ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
-void launch_prep_keys(const uint32_t* in, uint64_t n, uint64_t K, uint32_t* out, DevState* st,
-                      bool allow_nokey, int sms, cudaStream_t stream) {
-  if (n == 0) return;
-  uint64_t b = (n + kThreads - 1) / kThreads;
-  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
-  note_launches(1);
-  prep_keys_kernel<<<(unsigned)b, kThreads, 0, stream>>>(in, n, K, out, st, allow_nokey ? 1 : 0);
-}
-
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream) {
   if (n == 0) return;
@@ -881,7 +936,7 @@ uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms) {
   // longest chunk (<= kPushSpan / groups per block, >= 8) that still gives
   // every SM four blocks of work
   uint64_t ch = 0;
-  dispatch_gc(D / 4, [&](auto Gc, auto) {
+  dispatch_push_gc(D / 4, [&](auto Gc, auto) {
     constexpr int G = decltype(Gc)::value;
     constexpr uint64_t NG = kThreads / G;
     ch = kPushSpan / NG;
@@ -895,7 +950,7 @@ uint64_t push_long_part_rows(uint64_t nspans) { return nspans / kLongSub + nspan
 
 uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk) {
   uint64_t span = 0;
-  dispatch_gc(D / 4, [&](auto Gc, auto) {
+  dispatch_push_gc(D / 4, [&](auto Gc, auto) {
     constexpr int G = decltype(Gc)::value;
     span = chunk * (kThreads / G);
   });
@@ -904,7 +959,7 @@ uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk) {
 
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream) {
   if (a.n == 0) return;
-  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+  dispatch_push_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     constexpr int R = 2 / C > 0 ? 2 / C : 1;
     uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
@@ -930,10 +985,10 @@ void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlist
     if (b == 0) continue;
     note_launches(1);
     events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(lists[i].keys, lists[i].count,
-                                                            lists[i].sign, s.ev_delta);
+                                                            lists[i].sign, s.ev_delta, s.st);
   }
   for (int i = 0; i < nlists; ++i) {
-    uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
+    uint64_t b = (lists[i].cap + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
     if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
     if (b == 0) continue;
     note_launches(1);
@@ -947,7 +1002,8 @@ void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list
                          cudaStream_t stream) {
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    const unsigned grid = grid_for(max_events, G, sms);
+    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // keys per group, as in the kernels
+    const unsigned grid = grid_for((max_events + R - 1) / R, G, sms);
     note_launches(3);
     evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list);
     alloc_kernel<<<1, 1, 0, stream>>>(s.st, (int32_t)s.S);

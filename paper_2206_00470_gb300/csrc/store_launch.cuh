@@ -44,8 +44,6 @@ struct EventList {
   int sign;
 };
 
-void launch_prep_keys(const uint32_t* in, uint64_t n, uint64_t K, uint32_t* out, DevState* st,
-                      bool allow_nokey, int sms, cudaStream_t stream);
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream);
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream);
