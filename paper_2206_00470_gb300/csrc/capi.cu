@@ -238,20 +238,17 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
                ctx->sms, ctx->dstate, &ctx->bar_base, ctx->stream, &sk, &sp));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
-  const uint64_t nspans = push_spans(ctx->s.D, n, chunk);
-  float *ph = nullptr, *pt = nullptr, *bh = nullptr, *bt = nullptr;
+  float *ph = nullptr, *pt = nullptr;
   uint32_t* longs = nullptr;
   CK(pool_alloc(ctx, &ph, nchunks * ctx->s.D));
   CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
-  CK(pool_alloc(ctx, &bh, nspans * ctx->s.D));
-  CK(pool_alloc(ctx, &bt, nspans * ctx->s.D));
   float* lparts = nullptr;
-  CK(pool_alloc(ctx, &longs, push_long_list_words(nspans)));
-  CK(pool_alloc(ctx, &lparts, push_long_part_rows(nspans) * ctx->s.D));
+  CK(pool_alloc(ctx, &longs, push_long_list_words(nchunks)));
+  CK(pool_alloc(ctx, &lparts, push_long_part_rows(nchunks) * ctx->s.D));
   CK(cudaMemsetAsync(longs, 0, sizeof(uint32_t), ctx->stream));
   CK(cudaMemsetAsync(&ctx->dstate->last_unique, 0, sizeof(uint32_t), ctx->stream));
   ctx->push_rows_host += n;
-  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, bh, bt, longs + 1, longs, lparts};
+  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, longs + 1, longs, lparts};
   {
     ProfScope ps(ctx, 6);
     launch_push(ctx->s, a, ctx->sms, ctx->stream);
@@ -263,8 +260,6 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   pool_free(ctx, hist);
   pool_free(ctx, ph);
   pool_free(ctx, pt);
-  pool_free(ctx, bh);
-  pool_free(ctx, bt);
   pool_free(ctx, longs);
   pool_free(ctx, lparts);
   return check_launch(ctx, "push");

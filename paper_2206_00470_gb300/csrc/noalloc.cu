@@ -59,15 +59,14 @@ bool is_device_ptr(const void* p) {
 
 // Byte offsets of the scratch regions of one push of n rows.
 struct Layout {
-  size_t ka, kb, va, vb, hist, ph, pt, bh, bt, longs, lparts, total;
-  uint64_t chunk, nchunks, nspans;
+  size_t ka, kb, va, vb, hist, ph, pt, longs, lparts, total;
+  uint64_t chunk, nchunks;
 };
 
 Layout layout(uint32_t D, uint64_t n, int sms) {
   Layout L{};
   L.chunk = adapm::push_chunk_rows(D, n, sms);
   L.nchunks = (n + L.chunk - 1) / L.chunk;
-  L.nspans = adapm::push_spans(D, n, L.chunk);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t at = off;
@@ -81,10 +80,8 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   L.hist = take(adapm::sort_scratch_words(n) * 4);
   L.ph = take(L.nchunks * D * 4);
   L.pt = take(L.nchunks * D * 4);
-  L.bh = take(L.nspans * D * 4);
-  L.bt = take(L.nspans * D * 4);
-  L.longs = take(adapm::push_long_list_words(L.nspans) * 4);
-  L.lparts = take(adapm::push_long_part_rows(L.nspans) * D * 4);
+  L.longs = take(adapm::push_long_list_words(L.nchunks) * 4);
+  L.lparts = take(adapm::push_long_part_rows(L.nchunks) * D * 4);
   L.total = off;
   return L;
 }
@@ -161,8 +158,6 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
              L.chunk,
              L.nchunks,
              worker,
-             reinterpret_cast<float*>(base + L.bh),
-             reinterpret_cast<float*>(base + L.bt),
              longs + 1,
              longs,
              reinterpret_cast<float*>(base + L.lparts)};

@@ -322,16 +322,16 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     const uint32_t nmask = (1u << nnbits) - 1u;
     uint32_t* tcur = (p & 1) ? table1 : table0;
     uint32_t* tnext = (p & 1) ? table0 : table1;
-    // 1. exclusive prefix of each digit over the chunks, digit totals, and
-    // the digit's row of the next pass's table cleared.  Up to 16 chunks: one
-    // thread per digit (its row in one round of loads); more: one warp per
-    // digit, its row read in batches of 256 chunks, eight independent
-    // coalesced loads per lane
+    // 1. exclusive prefix of each digit over the chunks and digit totals.
+    // Up to 16 chunks: one thread per digit (its row in one round of
+    // loads); more: one warp per digit, its row read in batches of 512 (256
+    // with positions) chunks, one coalesced load per lane and 32 chunks, all
+    // of a batch issued together.  Every block
+    // also clears its own column of the next pass's table.
+    if (more)
+      for (uint32_t d = threadIdx.x; d <= nmask; d += kSortThreads) tnext[(uint64_t)d * B + b] = 0u;
     if (B <= 16) {
-      for (uint32_t d = b * kSortThreads + threadIdx.x; d < kDigits; d += B * kSortThreads) {
-        if (more && d <= nmask)
-          for (uint32_t j = 0; j < B; ++j) tnext[(uint64_t)d * B + j] = 0u;
-        if (d > mask) continue;
+      for (uint32_t d = b * kSortThreads + threadIdx.x; d <= mask; d += B * kSortThreads) {
         uint32_t* row = tcur + (uint64_t)d * B;
         uint32_t v[16];
 #pragma unroll
@@ -345,21 +345,20 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
         a.totals[d] = run;
       }
     } else {
-      for (uint32_t d = b * kWarps + warp; d < kDigits; d += B * kWarps) {
-        if (more && d <= nmask)
-          for (uint32_t j = lane; j < B; j += 32) tnext[(uint64_t)d * B + j] = 0u;
-        if (d > mask) continue;
+      // (the first pass's ranks stay in registers with positions: a smaller batch)
+      constexpr int QB = POS ? 8 : 16;
+      for (uint32_t d = b * kWarps + warp; d <= mask; d += B * kWarps) {
         uint32_t* row = tcur + (uint64_t)d * B;
         uint32_t carry = 0;
-        for (uint32_t j0 = 0; j0 < B; j0 += 256) {
-          uint32_t v[8];
+        for (uint32_t j0 = 0; j0 < B; j0 += 32 * QB) {
+          uint32_t v[QB];
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
+          for (int q = 0; q < QB; ++q) {
             const uint32_t j = j0 + q * 32 + lane;
             v[q] = j < B ? __ldcg(row + j) : 0u;
           }
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
+          for (int q = 0; q < QB; ++q) {
             uint32_t x = v[q];
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {

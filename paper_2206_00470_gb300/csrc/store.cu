@@ -33,6 +33,34 @@ __device__ __forceinline__ float4 f4add(float4 a, float4 b) {
 }
 __device__ __forceinline__ float4 f4zero() { return make_float4(0.f, 0.f, 0.f, 0.f); }
 
+// Block-wide sums of two per-thread counts, returned to thread 0 (every
+// thread of the block calls it), so that a kernel adds its statistics to
+// DevState with one atomic per block instead of one per thread: thousands of
+// atomics on the one line of DevState would queue up in its L2 slice, in
+// front of the row traffic that the slice also serves.
+__device__ __forceinline__ void block_sum2(uint32_t& a, uint32_t& b) {
+  __shared__ uint32_t wa[32], wb[32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
+    b += __shfl_xor_sync(0xFFFFFFFFu, b, o);
+  }
+  const int warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    wa[warp] = a;
+    wb[warp] = b;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    a = 0;
+    b = 0;
+    for (int w = 0; w < nw; ++w) {
+      a += wa[w];
+      b += wb[w];
+    }
+  }
+}
+
 template <int G>
 __device__ __forceinline__ uint64_t group_id() {
   return ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
@@ -113,37 +141,20 @@ __device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, u
   }
 }
 
-// tot += rows first..last of a piece array (ascending, loads issued in batches)
-template <int G, int C>
-__device__ __forceinline__ void sum_pieces(float4 (&tot)[C], const float4* pieces, uint64_t first,
-                                           uint64_t last, uint32_t D4, int lane) {
-  constexpr int UB = 8 / C > 0 ? 8 / C : 1;
-  for (uint64_t m0 = first; m0 <= last; m0 += UB) {
-    float4 t[UB][C];
-#pragma unroll
-    for (int u = 0; u < UB; ++u)
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        t[u][c] = (m0 + u <= last && col < D4) ? pieces[(m0 + u) * D4 + col] : f4zero();
-      }
-#pragma unroll
-    for (int u = 0; u < UB; ++u)
-      if (m0 + u <= last)
-#pragma unroll
-        for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
-  }
-}
-
-// Each block stages kPushSpan consecutive sorted positions (keys and source
-// positions) in shared memory; its groups own consecutive chunks of them.
-constexpr int kPushSpan = 1024;
+// Each block stages a span of up to kPushSpan consecutive sorted positions
+// (keys and source positions) in shared memory; its groups own consecutive
+// chunks of it.  A segment cut by chunk boundaries leaves a partial sum per
+// chunk (a tail piece in the chunk it starts in, head pieces in the chunks
+// it continues into); push_fixup / push_long add the pieces up.
+constexpr int kPushSpan = 3072;
+// resident push_chunks blocks per SM (its launch bounds)
+constexpr int push_blocks_per_sm(int C) { return C >= 4 ? 2 : 3; }
 // a segment cut by chunk boundaries and spanning at most this many further
 // chunks is combined by one group; longer ones (hot keys) by a whole block
 constexpr int kShortSpan = 8;
 
 template <int G, int C, int R>
-__global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 4) push_chunks_kernel(Store s, PushArgs a) {
+__global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_kernel(Store s, PushArgs a) {
   if (sort_failed(s.st)) return;
   constexpr int NG = kThreads / G;
   const uint32_t CH = (uint32_t)a.chunk;            // rows per group, NG * CH <= kPushSpan
@@ -265,73 +276,10 @@ __global__ void __launch_bounds__(kThreads, C >= 4 ? 2 : 4) push_chunks_kernel(S
         }
       }
     }
-    // combine the chunk pieces inside this span: a segment begun in chunk gi
-    // that ends later in the span is applied here; one that leaves the span
-    // leaves a span tail piece, and the span's first segment, begun before
-    // the span, a span head piece (both combined across spans by the fix-up)
-    __syncthreads();
-    const uint64_t b = P0 / span;
-    const uint64_t jb = P0 / CH;
-    if (p0 < p1) {
-      const uint32_t kl = sk[1 + p1 - 1];
-      const bool started = (P0 + p0 == 0) || sk[p0] != kl;
-      const bool cont = (P0 + p1 < a.n) && sk[1 + p1] == kl;
-      if (kl != kNoKey && started && cont) {
-        uint32_t q = p1, g_last = gi;
-        bool leaves = false;
-        while (true) {
-          if (q == len) {
-            leaves = true;
-            break;
-          }
-          ++g_last;
-          const uint32_t qe = q + CH < len ? q + CH : len;
-          if (P0 + qe < a.n && sk[1 + qe] == kl) {
-            q = qe;
-            continue;
-          }
-          break;
-        }
-        float4 tot[C];
-#pragma unroll
-        for (int c = 0; c < C; ++c) {
-          const uint32_t col = lane + c * G;
-          tot[c] = col < D4 ? pt4[(jb + gi) * D4 + col] : f4zero();
-        }
-        sum_pieces<G, C>(tot, ph4, jb + gi + 1, jb + g_last, D4, lane);
-        if (leaves) {
-          float4* bt4 = reinterpret_cast<float4*>(a.span_tail);
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + c * G;
-            if (col < D4) bt4[b * D4 + col] = tot[c];
-          }
-        } else {
-          apply_sum<C>(s, mapw, kl, tot, lane, G);
-        }
-      }
-    }
-    if (gi == 0 && P0 > 0 && sk[1] == sk[0] && sk[1] != kNoKey) {
-      const uint32_t kf = sk[1];
-      uint32_t g_last = 0;
-      uint32_t qe = CH < len ? CH : len;
-      while (qe < len && P0 + qe < a.n && sk[1 + qe] == kf) {
-        ++g_last;
-        qe = qe + CH < len ? qe + CH : len;
-      }
-      float4 tot[C];
-#pragma unroll
-      for (int c = 0; c < C; ++c) tot[c] = f4zero();
-      sum_pieces<G, C>(tot, ph4, jb, jb + g_last, D4, lane);
-      float4* bh4 = reinterpret_cast<float4*>(a.span_head);
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        if (col < D4) bh4[b * D4 + col] = tot[c];
-      }
-    }
   }
-  if (heads) {
+  uint32_t unused = 0;
+  block_sum2(heads, unused);
+  if (threadIdx.x == 0 && heads) {
     atomicAdd(&s.st->last_unique, heads);
     atomicAdd(&s.st->push_unique, (unsigned long long)heads);
   }
@@ -513,31 +461,60 @@ __global__ void events_add_kernel(const uint32_t* __restrict__ keys, const uint3
     atomicAdd(ev_delta + keys[i], sign);
 }
 
-__device__ __forceinline__ uint32_t lanemask_lt_() {
-  uint32_t m;
-  asm("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
-  return m;
-}
-
-// warp-aggregated append to a device list
-__device__ __forceinline__ void warp_append(bool want, uint32_t value, uint32_t* counter, uint32_t* list) {
-  const uint32_t m = __ballot_sync(0xFFFFFFFFu, want);
-  if (m == 0) return;
-  const int leader = __ffs(m) - 1;
-  uint32_t base = 0;
-  if ((int)(threadIdx.x & 31) == leader) base = atomicAdd(counter, (uint32_t)__popc(m));
-  base = __shfl_sync(0xFFFFFFFFu, base, leader);
-  if (want) list[base + __popc(m & lanemask_lt_())] = value;
+// Exclusive block-wide scans of two per-thread counts (every thread of the
+// block calls it); ta / tb receive the block totals.
+__device__ __forceinline__ void block_exclusive_scan2(uint32_t& a, uint32_t& b, uint32_t& ta, uint32_t& tb) {
+  __shared__ uint32_t sa[32], sb[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  uint32_t xa = a, xb = b;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, xa, o);
+    const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, xb, o);
+    if (lane >= o) {
+      xa += ya;
+      xb += yb;
+    }
+  }
+  if (lane == 31) {
+    sa[warp] = xa;
+    sb[warp] = xb;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t va = lane < nw ? sa[lane] : 0u, vb = lane < nw ? sb[lane] : 0u;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, va, o);
+      const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, vb, o);
+      if (lane >= o) {
+        va += ya;
+        vb += yb;
+      }
+    }
+    if (lane < nw) {
+      sa[lane] = va;
+      sb[lane] = vb;
+    }
+  }
+  __syncthreads();
+  a = (warp > 0 ? sa[warp - 1] : 0u) + xa - a;
+  b = (warp > 0 ? sb[warp - 1] : 0u) + xb - b;
+  ta = sa[nw - 1];
+  tb = sb[nw - 1];
+  __syncthreads();
 }
 
 // Net refcount change of every listed key (4 keys per thread per round, each
 // step a round of independent accesses), appended to the create list (0 ->
-// >0) or the evict list (>0 -> 0, if a replica exists).
+// >0) or the evict list (>0 -> 0, if a replica exists).  The order of a list
+// is not specified.
 __global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys,
                                     const uint32_t* __restrict__ count, uint32_t* create_list,
                                     uint32_t* evict_list) {
   if (sort_failed(s.st)) return;
   constexpr int Q = 4;
+  __shared__ uint32_t base_s[2];
   const uint32_t n = *count;
   uint16_t* rcw = s.rc + (uint64_t)w * s.K;
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
@@ -577,11 +554,28 @@ __global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restr
 #pragma unroll
     for (int q = 0; q < Q; ++q)
       if (evict[q]) evict[q] = mapw[k[q]] >= 0;
+    // append: block-wide offsets, one atomic per list per block and round
+    uint32_t oc = 0, oe = 0;
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
-      warp_append(create[q], k[q], &s.st->n_create, create_list);
-      warp_append(evict[q], k[q], &s.st->n_evict, evict_list);
+      oc += create[q] ? 1u : 0u;
+      oe += evict[q] ? 1u : 0u;
     }
+    uint32_t tc, te;
+    block_exclusive_scan2(oc, oe, tc, te);
+    if (threadIdx.x == 0) {
+      base_s[0] = tc ? atomicAdd(&s.st->n_create, tc) : 0u;
+      base_s[1] = te ? atomicAdd(&s.st->n_evict, te) : 0u;
+    }
+    __syncthreads();
+    oc += base_s[0];
+    oe += base_s[1];
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      if (create[q]) create_list[oc++] = k[q];
+      if (evict[q]) evict_list[oe++] = k[q];
+    }
+    __syncthreads();
   }
 }
 
@@ -837,7 +831,8 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
       }
     }
   }
-  if (lane == 0 && nkeys) {
+  block_sum2(nkeys, nreps);
+  if (threadIdx.x == 0 && nkeys) {
     atomicAdd(&s.st->sync_keys, (unsigned long long)nkeys);
     atomicAdd(&s.st->sync_replicas, (unsigned long long)nreps);
   }
@@ -933,47 +928,35 @@ void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float*
 }
 
 uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms) {
-  // longest chunk (<= kPushSpan / groups per block, >= 8) that still gives
-  // every SM four blocks of work
+  // one span per resident block where the span fits in shared memory: rows
+  // per group = n / (groups per block x resident blocks), in [8, kPushSpan / groups]
   uint64_t ch = 0;
-  dispatch_push_gc(D / 4, [&](auto Gc, auto) {
-    constexpr int G = decltype(Gc)::value;
+  dispatch_push_gc(D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     constexpr uint64_t NG = kThreads / G;
-    ch = kPushSpan / NG;
-    while (ch > 8 && n / (ch * NG) < (uint64_t)sms * 4) ch /= 2;
+    const uint64_t groups = NG * (uint64_t)sms * push_blocks_per_sm(C);
+    ch = (n + groups - 1) / groups;
+    if (ch < 8) ch = 8;
+    if (ch > kPushSpan / NG) ch = kPushSpan / NG;
   });
   return ch;
 }
 
-uint64_t push_long_list_words(uint64_t nspans) { return 4 * (nspans / 8 + 2) + 1; }
-uint64_t push_long_part_rows(uint64_t nspans) { return nspans / kLongSub + nspans / 8 + 2; }
-
-uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk) {
-  uint64_t span = 0;
-  dispatch_push_gc(D / 4, [&](auto Gc, auto) {
-    constexpr int G = decltype(Gc)::value;
-    span = chunk * (kThreads / G);
-  });
-  return (n + span - 1) / span;
-}
+uint64_t push_long_list_words(uint64_t nchunks) { return 4 * (nchunks / 8 + 2) + 1; }
+uint64_t push_long_part_rows(uint64_t nchunks) { return nchunks / kLongSub + nchunks / 8 + 2; }
 
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream) {
   if (a.n == 0) return;
   dispatch_push_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    constexpr int R = 2 / C > 0 ? 2 / C : 1;
-    uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
-    const uint64_t cap = (uint64_t)sms * 4;
+    constexpr int R = 4 / C > 0 ? 4 / C : 1;
+    // one block per span: the block scheduler balances spans over the SMs
+    const uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
     note_launches(3);
-    push_chunks_kernel<G, C, R><<<(unsigned)(spans < cap ? spans : cap), kThreads, 0, stream>>>(s, a);
-    PushArgs sp = a;                       // the fix-up works on span pieces
-    sp.part_head = a.span_head;
-    sp.part_tail = a.span_tail;
-    sp.chunk = a.chunk * (kThreads / G);
-    sp.nchunks = spans;
-    push_fixup_kernel<G, C><<<grid_for(sp.nchunks, G, sms), kThreads, 0, stream>>>(s, sp, a.long_list,
-                                                                                  a.long_count);
-    push_long_kernel<G, C><<<(unsigned)sms * 2, kThreads, 0, stream>>>(s, sp, a.long_list, a.long_count);
+    push_chunks_kernel<G, C, R><<<(unsigned)spans, kThreads, 0, stream>>>(s, a);
+    push_fixup_kernel<G, C><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a, a.long_list,
+                                                                                 a.long_count);
+    push_long_kernel<G, C><<<(unsigned)sms * 2, kThreads, 0, stream>>>(s, a, a.long_list, a.long_count);
   });
 }
 

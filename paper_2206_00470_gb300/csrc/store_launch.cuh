@@ -18,19 +18,14 @@ struct PushArgs {
   uint64_t chunk;
   uint64_t nchunks;
   uint32_t worker;
-  float* span_head;       // pieces per block span (groups x chunk rows): nspans x D floats
-  float* span_tail;
-  uint32_t* long_list;    // push_long_list_words(nspans) - 1 words of scratch
+  uint32_t* long_list;    // push_long_list_words(nchunks) - 1 words of scratch
   uint32_t* long_count;   // one word, zeroed by the caller
-  float* long_parts;      // push_long_part_rows(nspans) x D floats of scratch
+  float* long_parts;      // push_long_part_rows(nchunks) x D floats of scratch
 };
 
-// Scratch sizes of the hot-key (long segment) combine for nspans block spans.
-uint64_t push_long_list_words(uint64_t nspans);
-uint64_t push_long_part_rows(uint64_t nspans);
-
-// Number of block spans of a push of n rows with chunk length `chunk`.
-uint64_t push_spans(uint32_t D, uint64_t n, uint64_t chunk);
+// Scratch sizes of the hot-key (long segment) combine for nchunks chunks.
+uint64_t push_long_list_words(uint64_t nchunks);
+uint64_t push_long_part_rows(uint64_t nchunks);
 
 // Rows per push chunk for value length D and a batch of n rows.
 uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms);
