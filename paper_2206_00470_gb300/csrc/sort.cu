@@ -45,6 +45,7 @@ constexpr int kDPT = kDigits / kSortThreads;       // digits per thread (2)
 constexpr uint32_t kMaxSortBlocks = 4096;
 constexpr uint32_t kSpinLimit = 1u << 21;          // polls of one barrier wait
 constexpr int kScratchHead = 32;                   // words before the totals
+constexpr int kScanQ = 5;                          // digit-row entries per lane, four warps a row
 
 constexpr int kCompactItems = 8;                   // compaction: keys per thread
 constexpr int kTile = kSortThreads * kCompactItems;
@@ -324,9 +325,9 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     uint32_t* tnext = (p & 1) ? table0 : table1;
     // 1. exclusive prefix of each digit over the chunks and digit totals.
     // Up to 16 chunks: one thread per digit (its row in one round of
-    // loads); more: one warp per digit, its row read in batches of 512 (256
-    // with positions) chunks, one coalesced load per lane and 32 chunks, all
-    // of a batch issued together.  Every block
+    // loads); 129 to 640: four warps per digit row, a quarter each in one
+    // round of coalesced loads, combined through shared memory; otherwise
+    // one warp per digit row, read in batches.  Every block
     // also clears its own column of the next pass's table.
     if (more)
       for (uint32_t d = threadIdx.x; d <= nmask; d += kSortThreads) tnext[(uint64_t)d * B + b] = 0u;
@@ -343,6 +344,47 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
           run += v[j];
         }
         a.totals[d] = run;
+      }
+    } else if (B > 128 && B <= 4 * 32 * kScanQ) {
+      // four warps per digit row (a quarter each, kept in registers), two
+      // rows per block at a time
+      const uint32_t half = warp >> 2, quarter = warp & 3;
+      const uint32_t seg = (B + 3) / 4;
+      const uint32_t jb = quarter * seg;
+      const uint32_t je = jb + seg < B ? jb + seg : B;
+      for (uint32_t dp = b; dp * 2 <= mask; dp += B) {   // block-uniform trip count
+        const uint32_t d = dp * 2 + half;
+        const bool act = d <= mask;
+        uint32_t* row = tcur + (uint64_t)d * B;
+        uint32_t v[kScanQ], x[kScanQ];
+#pragma unroll
+        for (int q = 0; q < kScanQ; ++q) {
+          const uint32_t j = jb + q * 32 + lane;
+          v[q] = act && j < je ? __ldcg(row + j) : 0u;
+        }
+        uint32_t carry = 0;
+#pragma unroll
+        for (int q = 0; q < kScanQ; ++q) {
+          uint32_t y = v[q];
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, y, o);
+            if (lane >= o) y += t;
+          }
+          x[q] = carry + y - v[q];   // exclusive within the quarter
+          carry += __shfl_sync(0xFFFFFFFFu, y, 31);
+        }
+        if (lane == 0) sm.scan[warp] = carry;
+        __syncthreads();
+        uint32_t before = 0;
+        for (uint32_t w2 = 0; w2 < quarter; ++w2) before += sm.scan[half * 4 + w2];
+#pragma unroll
+        for (int q = 0; q < kScanQ; ++q) {
+          const uint32_t j = jb + q * 32 + lane;
+          if (act && j < je) row[j] = before + x[q];
+        }
+        if (act && quarter == 3 && lane == 0) a.totals[d] = before + carry;
+        __syncthreads();
       }
     } else {
       // (the first pass's ranks stay in registers with positions: a smaller batch)

@@ -73,6 +73,9 @@ __device__ __forceinline__ uint64_t group_count() {
 // ---------------------------------------------------------------------------
 // pull (and main-only gather for inspection when w < 0)
 // ---------------------------------------------------------------------------
+// R rows per group and round, software-pipelined so that one round issues
+// the row loads of round i, the slot lookups of round i+1 and the key loads
+// of round i+2 together: one memory latency per round instead of three.
 template <int G, int C, int R>
 __global__ void __launch_bounds__(kThreads)
 pull_kernel(Store s, int w, const uint32_t* __restrict__ keys, uint64_t n, float* __restrict__ out) {
@@ -83,32 +86,56 @@ pull_kernel(Store s, int w, const uint32_t* __restrict__ keys, uint64_t n, float
   const float4* val4 = reinterpret_cast<const float4*>(s.val);
   float4* out4 = reinterpret_cast<float4*>(out);
   const int32_t* mapw = w >= 0 ? s.map + (uint64_t)w * s.K : nullptr;
+  const uint64_t step = ng * R;
   bool bad = false;
-  for (uint64_t base = g * R; base < n; base += ng * R) {
-    uint32_t k[R];
+  auto load_keys = [&](uint64_t b, uint32_t (&k)[R]) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) k[r] = base + r < n ? __ldg(keys + base + r) : kNoKey;
-    int32_t sl[R];
+    for (int r = 0; r < R; ++r) k[r] = b + r < n ? __ldg(keys + b + r) : kNoKey;
+  };
+  auto load_slots = [&](const uint32_t (&k)[R], int32_t (&sl)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) sl[r] = (mapw != nullptr && k[r] < s.K) ? __ldg(mapw + k[r]) : -1;
+  };
+  uint64_t base = g * R;
+  uint32_t k0[R], k1[R];
+  int32_t sl0[R];
+  load_keys(base, k0);
+  load_keys(base + step, k1);
+  load_slots(k0, sl0);
+  for (; base < n; base += step) {
+    // this round's rows
     const float4* src[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       src[r] = nullptr;
-      if (k[r] < s.K) src[r] = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
+      if (k0[r] < s.K) src[r] = sl0[r] >= 0 ? val4 + (uint64_t)sl0[r] * D4 : main4 + (uint64_t)k0[r] * D4;
       else if (base + r < n) bad = true;
     }
+    float4 v[R][C];
 #pragma unroll
     for (int c = 0; c < C; ++c) {
       const uint32_t col = lane + c * G;
-      if (col < D4) {
-        float4 v[R];
 #pragma unroll
-        for (int r = 0; r < R; ++r) v[r] = src[r] != nullptr ? __ldg(src[r] + col) : f4zero();
+      for (int r = 0; r < R; ++r) v[r][c] = (src[r] != nullptr && col < D4) ? __ldg(src[r] + col) : f4zero();
+    }
+    // next round's slots and the keys of the round after
+    int32_t sl1[R];
+    uint32_t k2[R];
+    load_slots(k1, sl1);
+    load_keys(base + 2 * step, k2);
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const uint32_t col = lane + c * G;
+      if (col < D4)
 #pragma unroll
         for (int r = 0; r < R; ++r)
-          if (base + r < n) __stcs(out4 + (base + r) * D4 + col, v[r]);
-      }
+          if (base + r < n) __stcs(out4 + (base + r) * D4 + col, v[r][c]);
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      k0[r] = k1[r];
+      sl0[r] = sl1[r];
+      k1[r] = k2[r];
     }
   }
   if (bad && lane == 0) set_error(s.st, ERR_KEY_RANGE);
@@ -366,6 +393,7 @@ __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs 
 // piece and the item sums in item order and applies the total.  Every sum has
 // a fixed order, so the result does not depend on which block finishes last.
 constexpr uint32_t kLongSub = 32;
+constexpr uint32_t kLongSmem = 1024;   // long-list entries whose item bases sit in shared memory
 
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a, uint32_t* long_list,
@@ -383,21 +411,68 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
   float4* lp4 = reinterpret_cast<float4*>(a.long_parts);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   const uint32_t nl = *long_count;
+  // item bases of the first kLongSmem entries (block scan of their item
+  // counts), so that locating an item is a binary search in shared memory
+  __shared__ uint32_t s_base[kLongSmem + 1];
+  __shared__ uint32_t s_scan[kThreads / 32];
+  const uint32_t ns_tab = nl < kLongSmem ? nl : kLongSmem;
+  {
+    uint32_t carry = 0;
+    for (uint32_t e0 = 0; e0 < ns_tab; e0 += kThreads) {   // block-uniform trip count
+      const uint32_t e = e0 + threadIdx.x;
+      const uint32_t cnt = e < ns_tab ? (long_list[4 * e + 1] - long_list[4 * e] + kLongSub - 1) / kLongSub : 0u;
+      uint32_t x = cnt;
+      const int ln = threadIdx.x & 31, wp = threadIdx.x >> 5;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (ln >= o) x += y;
+      }
+      if (ln == 31) s_scan[wp] = x;
+      __syncthreads();
+      uint32_t before = 0, total = 0;
+      for (int w2 = 0; w2 < kThreads / 32; ++w2) {
+        if (w2 < wp) before += s_scan[w2];
+        total += s_scan[w2];
+      }
+      if (e < ns_tab) s_base[e] = carry + before + x - cnt;
+      carry += total;
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) s_base[ns_tab] = carry;
+    __syncthreads();
+  }
   for (uint64_t q = blockIdx.x;; q += gridDim.x) {
     // locate work item q: entry e, item it, first item of the entry `base`
     uint64_t base = 0, it = 0, ns = 0, j = 0, m_end = 0;
     uint32_t e = 0;
-    for (; e < nl; ++e) {
+    if (q < s_base[ns_tab]) {
+      uint32_t lo = 0, hi = ns_tab - 1;   // last entry whose base <= q
+      while (lo < hi) {
+        const uint32_t mid = (lo + hi + 1) / 2;
+        if (s_base[mid] <= q) lo = mid; else hi = mid - 1;
+      }
+      e = lo;
+      base = s_base[e];
       j = long_list[4 * e];
       m_end = long_list[4 * e + 1];
       ns = (m_end - j + kLongSub - 1) / kLongSub;
-      if (q < base + ns) {
-        it = q - base;
-        break;
+      it = q - base;
+    } else {
+      // entries past the table: walk them
+      base = s_base[ns_tab];
+      for (e = ns_tab; e < nl; ++e) {
+        j = long_list[4 * e];
+        m_end = long_list[4 * e + 1];
+        ns = (m_end - j + kLongSub - 1) / kLongSub;
+        if (q < base + ns) {
+          it = q - base;
+          break;
+        }
+        base += ns;
       }
-      base += ns;
+      if (e == nl) break;
     }
-    if (e == nl) break;
     const uint64_t lo = j + 1 + it * kLongSub;
     const uint64_t hi = lo + kLongSub - 1 < m_end ? lo + kLongSub - 1 : m_end;
     float4 acc[C];
@@ -441,8 +516,23 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
         tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
-        for (uint64_t i2 = 0; i2 < ns; ++i2)
-          if (col < D4) tot[c] = f4add(tot[c], __ldcg(lp4 + (base + i2) * D4 + col));
+      }
+      // the item sums in item order, several loads in flight
+      constexpr int UB = 8 / C > 0 ? 8 / C : 1;
+      for (uint64_t i0 = 0; i0 < ns; i0 += UB) {
+        float4 t[UB][C];
+#pragma unroll
+        for (int u = 0; u < UB; ++u)
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            t[u][c] = (i0 + u < ns && col < D4) ? __ldcg(lp4 + (base + i0 + u) * D4 + col) : f4zero();
+          }
+#pragma unroll
+        for (int u = 0; u < UB; ++u)
+          if (i0 + u < ns)
+#pragma unroll
+            for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
       }
       apply_sum<C>(s, mapw, kl, tot, lane, G);
     }
