@@ -214,7 +214,6 @@ adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventLis
   uint32_t *create_list = nullptr, *evict_list = nullptr;
   CK(pool_alloc(ctx, &create_list, total));
   CK(pool_alloc(ctx, &evict_list, total));
-  CK(cudaMemsetAsync(&ctx->dstate->n_create, 0, 2 * sizeof(uint32_t), ctx->stream));
   launch_events(ctx->s, w, ev.data(), (int)ev.size(), create_list, evict_list, ctx->sms, ctx->stream);
   launch_evict_create(ctx->s, w, create_list, evict_list, total, ctx->sms, ctx->stream);
   pool_free(ctx, create_list);

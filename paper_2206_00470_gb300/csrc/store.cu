@@ -543,12 +543,30 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
 // ---------------------------------------------------------------------------
 // intent events -> refcounts -> create / evict lists
 // ---------------------------------------------------------------------------
-__global__ void events_add_kernel(const uint32_t* __restrict__ keys, const uint32_t* __restrict__ count,
-                                  int sign, int32_t* __restrict__ ev_delta, const DevState* st) {
+// Up to kEventLists intent lists handled by one launch.
+constexpr int kEventLists = 8;
+struct EventBatch {
+  const uint32_t* keys[kEventLists];
+  const uint32_t* count[kEventLists];
+  int sign[kEventLists];
+  int n;
+};
+
+// ev_delta[k] += sign of every listed key; the first batch of an advance
+// also clears the create / evict list counters.
+__global__ void events_add_kernel(EventBatch eb, int32_t* __restrict__ ev_delta, DevState* st,
+                                  int clear_counts) {
+  if (clear_counts && blockIdx.x == 0 && threadIdx.x == 0) {
+    st->n_create = 0;
+    st->n_evict = 0;
+  }
   if (sort_failed(st)) return;
-  const uint32_t n = *count;
-  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
-    atomicAdd(ev_delta + keys[i], sign);
+  for (int l = 0; l < eb.n; ++l) {
+    const uint32_t n = *eb.count[l];
+    const uint32_t* keys = eb.keys[l];
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+      atomicAdd(ev_delta + keys[i], eb.sign[l]);
+  }
 }
 
 // Exclusive block-wide scans of two per-thread counts (every thread of the
@@ -599,73 +617,75 @@ __device__ __forceinline__ void block_exclusive_scan2(uint32_t& a, uint32_t& b, 
 // step a round of independent accesses), appended to the create list (0 ->
 // >0) or the evict list (>0 -> 0, if a replica exists).  The order of a list
 // is not specified.
-__global__ void events_apply_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys,
-                                    const uint32_t* __restrict__ count, uint32_t* create_list,
+__global__ void events_apply_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* create_list,
                                     uint32_t* evict_list) {
   if (sort_failed(s.st)) return;
   constexpr int Q = 4;
   __shared__ uint32_t base_s[2];
-  const uint32_t n = *count;
   uint16_t* rcw = s.rc + (uint64_t)w * s.K;
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
   const uint32_t stride = gridDim.x * blockDim.x * Q;
-  for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // warp-uniform trip count
-    uint32_t k[Q];
-    int32_t d[Q], old[Q];
+  for (int l = 0; l < eb.n; ++l) {
+    const uint32_t n = *eb.count[l];
+    const uint32_t* keys = eb.keys[l];
+    for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
+      uint32_t k[Q];
+      int32_t d[Q], old[Q];
 #pragma unroll
-    for (int q = 0; q < Q; ++q) {
-      const uint32_t i = b + q * blockDim.x + threadIdx.x;
-      k[q] = i < n ? keys[i] : 0u;
-    }
-#pragma unroll
-    for (int q = 0; q < Q; ++q) {
-      const uint32_t i = b + q * blockDim.x + threadIdx.x;
-      d[q] = i < n ? atomicExch(s.ev_delta + k[q], 0) : 0;
-    }
-#pragma unroll
-    for (int q = 0; q < Q; ++q) old[q] = d[q] != 0 ? (int32_t)rcw[k[q]] : 0;
-    bool create[Q], evict[Q];
-#pragma unroll
-    for (int q = 0; q < Q; ++q) {
-      create[q] = false;
-      evict[q] = false;
-      if (d[q] != 0) {
-        int32_t nw = old[q] + d[q];
-        if (nw < 0 || nw > 65535) {
-          set_error(s.st, ERR_REFCOUNT);
-          nw = nw < 0 ? 0 : 65535;
-        }
-        rcw[k[q]] = (uint16_t)nw;
-        create[q] = old[q] == 0 && nw > 0;
-        evict[q] = old[q] > 0 && nw == 0;
+      for (int q = 0; q < Q; ++q) {
+        const uint32_t i = b + q * blockDim.x + threadIdx.x;
+        k[q] = i < n ? keys[i] : 0u;
       }
-    }
-    // a key whose replica was never created (capacity exhausted) has nothing to destroy
 #pragma unroll
-    for (int q = 0; q < Q; ++q)
-      if (evict[q]) evict[q] = mapw[k[q]] >= 0;
-    // append: block-wide offsets, one atomic per list per block and round
-    uint32_t oc = 0, oe = 0;
+      for (int q = 0; q < Q; ++q) {
+        const uint32_t i = b + q * blockDim.x + threadIdx.x;
+        d[q] = i < n ? atomicExch(s.ev_delta + k[q], 0) : 0;
+      }
 #pragma unroll
-    for (int q = 0; q < Q; ++q) {
-      oc += create[q] ? 1u : 0u;
-      oe += evict[q] ? 1u : 0u;
-    }
-    uint32_t tc, te;
-    block_exclusive_scan2(oc, oe, tc, te);
-    if (threadIdx.x == 0) {
-      base_s[0] = tc ? atomicAdd(&s.st->n_create, tc) : 0u;
-      base_s[1] = te ? atomicAdd(&s.st->n_evict, te) : 0u;
-    }
-    __syncthreads();
-    oc += base_s[0];
-    oe += base_s[1];
+      for (int q = 0; q < Q; ++q) old[q] = d[q] != 0 ? (int32_t)rcw[k[q]] : 0;
+      bool create[Q], evict[Q];
 #pragma unroll
-    for (int q = 0; q < Q; ++q) {
-      if (create[q]) create_list[oc++] = k[q];
-      if (evict[q]) evict_list[oe++] = k[q];
+      for (int q = 0; q < Q; ++q) {
+        create[q] = false;
+        evict[q] = false;
+        if (d[q] != 0) {
+          int32_t nw = old[q] + d[q];
+          if (nw < 0 || nw > 65535) {
+            set_error(s.st, ERR_REFCOUNT);
+            nw = nw < 0 ? 0 : 65535;
+          }
+          rcw[k[q]] = (uint16_t)nw;
+          create[q] = old[q] == 0 && nw > 0;
+          evict[q] = old[q] > 0 && nw == 0;
+        }
+      }
+      // a key whose replica was never created (capacity exhausted) has nothing to destroy
+#pragma unroll
+      for (int q = 0; q < Q; ++q)
+        if (evict[q]) evict[q] = mapw[k[q]] >= 0;
+      // append: block-wide offsets, one atomic per list per block and round
+      uint32_t oc = 0, oe = 0;
+#pragma unroll
+      for (int q = 0; q < Q; ++q) {
+        oc += create[q] ? 1u : 0u;
+        oe += evict[q] ? 1u : 0u;
+      }
+      uint32_t tc, te;
+      block_exclusive_scan2(oc, oe, tc, te);
+      if (threadIdx.x == 0) {
+        base_s[0] = tc ? atomicAdd(&s.st->n_create, tc) : 0u;
+        base_s[1] = te ? atomicAdd(&s.st->n_evict, te) : 0u;
+      }
+      __syncthreads();
+      oc += base_s[0];
+      oe += base_s[1];
+#pragma unroll
+      for (int q = 0; q < Q; ++q) {
+        if (create[q]) create_list[oc++] = k[q];
+        if (evict[q]) evict_list[oe++] = k[q];
+      }
+      __syncthreads();
     }
-    __syncthreads();
   }
 }
 
@@ -801,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
 // sync
 // ---------------------------------------------------------------------------
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) sync_kernel(Store s) {
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint64_t hw = (uint64_t)s.st->high_water;
@@ -810,17 +830,26 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   uint32_t nkeys = 0, nreps = 0;
-  // R slots per group at a time: owners, holder masks, then (for keys held
-  // by one worker only, the common case) main and pending rows, each as one
-  // round of independent loads
+  // R slots per group at a time, software-pipelined: one round issues the
+  // main and pending rows of its slots (for keys held by one worker only,
+  // the common case), the holder masks of the next round's slots and the
+  // owners of the round after, so one memory latency per round
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
-  for (uint64_t b = g * R; b < hw; b += ng * R) {
-    unsigned long long own[R];
-    uint32_t mk[R];
+  const uint64_t step = ng * R;
+  auto load_owners = [&](uint64_t b0, unsigned long long (&o)[R]) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) own[r] = b + r < hw ? s.slot_owner[b + r] : kEmptySlot;
+    for (int r = 0; r < R; ++r) o[r] = b0 + r < hw ? s.slot_owner[b0 + r] : kEmptySlot;
+  };
+  auto load_holders = [&](const unsigned long long (&o)[R], uint32_t (&m)[R]) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) mk[r] = own[r] != kEmptySlot ? s.holders[(uint32_t)own[r]] : 0u;
+    for (int r = 0; r < R; ++r) m[r] = o[r] != kEmptySlot ? s.holders[(uint32_t)o[r]] : 0u;
+  };
+  unsigned long long own[R], own1[R];
+  uint32_t mk[R];
+  load_owners(g * R, own);
+  load_owners(g * R + step, own1);
+  load_holders(own, mk);
+  for (uint64_t b = g * R; b < hw; b += step) {
     bool single[R];
     float4 mv[R][C], av[R][C];
 #pragma unroll
@@ -835,6 +864,10 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
         av[r][c] = cv ? acc4[(b + r) * D4 + col] : f4zero();
       }
     }
+    uint32_t mk1[R];
+    unsigned long long own2[R];
+    load_holders(own1, mk1);
+    load_owners(b + 2 * step, own2);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       if (!single[r]) continue;
@@ -919,6 +952,12 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
           }
         }
       }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      own[r] = own1[r];
+      mk[r] = mk1[r];
+      own1[r] = own2[r];
     }
   }
   block_sum2(nkeys, nreps);
@@ -1052,21 +1091,30 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
 
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
                    uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
-  for (int i = 0; i < nlists; ++i) {
-    uint64_t b = (lists[i].cap + kThreads - 1) / kThreads;
-    if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
-    if (b == 0) continue;
-    note_launches(1);
-    events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(lists[i].keys, lists[i].count,
-                                                            lists[i].sign, s.ev_delta, s.st);
-  }
-  for (int i = 0; i < nlists; ++i) {
-    uint64_t b = (lists[i].cap + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
-    if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
-    if (b == 0) continue;
-    note_launches(1);
-    events_apply_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, lists[i].keys, lists[i].count,
-                                                              create_list, evict_list);
+  // lists in batches of kEventLists: all refcount deltas first, then the
+  // transitions (a key in several lists changes once, by its net delta)
+  const uint64_t cap_blocks = (uint64_t)sms * 8;
+  for (int pass = 0; pass < 2; ++pass) {
+    for (int i0 = 0; i0 < nlists; i0 += kEventLists) {
+      EventBatch eb{};
+      uint64_t cap = 0;
+      for (int l = 0; l < kEventLists && i0 + l < nlists; ++l) {
+        eb.keys[l] = lists[i0 + l].keys;
+        eb.count[l] = lists[i0 + l].count;
+        eb.sign[l] = lists[i0 + l].sign;
+        eb.n = l + 1;
+        if (lists[i0 + l].cap > cap) cap = lists[i0 + l].cap;
+      }
+      const uint64_t per = pass == 0 ? kThreads : 4 * kThreads;   // keys per block and round
+      uint64_t b = (cap + per - 1) / per;
+      if (b > cap_blocks) b = cap_blocks;
+      if (b == 0) b = 1;
+      note_launches(1);
+      if (pass == 0)
+        events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(eb, s.ev_delta, s.st, i0 == 0 ? 1 : 0);
+      else
+        events_apply_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list, evict_list);
+    }
   }
 }
 
