@@ -821,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
 // sync
 // ---------------------------------------------------------------------------
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) sync_kernel(Store s) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s) {
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint64_t hw = (uint64_t)s.st->high_water;
@@ -830,26 +830,17 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) sync_kernel(Store s)
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   uint32_t nkeys = 0, nreps = 0;
-  // R slots per group at a time, software-pipelined: one round issues the
-  // main and pending rows of its slots (for keys held by one worker only,
-  // the common case), the holder masks of the next round's slots and the
-  // owners of the round after, so one memory latency per round
+  // R slots per group at a time: owners, holder masks, then (for keys held
+  // by one worker only, the common case) main and pending rows, each as one
+  // round of independent loads
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
-  const uint64_t step = ng * R;
-  auto load_owners = [&](uint64_t b0, unsigned long long (&o)[R]) {
+  for (uint64_t b = g * R; b < hw; b += ng * R) {
+    unsigned long long own[R];
+    uint32_t mk[R];
 #pragma unroll
-    for (int r = 0; r < R; ++r) o[r] = b0 + r < hw ? s.slot_owner[b0 + r] : kEmptySlot;
-  };
-  auto load_holders = [&](const unsigned long long (&o)[R], uint32_t (&m)[R]) {
+    for (int r = 0; r < R; ++r) own[r] = b + r < hw ? s.slot_owner[b + r] : kEmptySlot;
 #pragma unroll
-    for (int r = 0; r < R; ++r) m[r] = o[r] != kEmptySlot ? s.holders[(uint32_t)o[r]] : 0u;
-  };
-  unsigned long long own[R], own1[R];
-  uint32_t mk[R];
-  load_owners(g * R, own);
-  load_owners(g * R + step, own1);
-  load_holders(own, mk);
-  for (uint64_t b = g * R; b < hw; b += step) {
+    for (int r = 0; r < R; ++r) mk[r] = own[r] != kEmptySlot ? s.holders[(uint32_t)own[r]] : 0u;
     bool single[R];
     float4 mv[R][C], av[R][C];
 #pragma unroll
@@ -864,10 +855,6 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) sync_kernel(Store s)
         av[r][c] = cv ? acc4[(b + r) * D4 + col] : f4zero();
       }
     }
-    uint32_t mk1[R];
-    unsigned long long own2[R];
-    load_holders(own1, mk1);
-    load_owners(b + 2 * step, own2);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       if (!single[r]) continue;
@@ -952,12 +939,6 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) sync_kernel(Store s)
           }
         }
       }
-    }
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      own[r] = own1[r];
-      mk[r] = mk1[r];
-      own1[r] = own2[r];
     }
   }
   block_sum2(nkeys, nreps);
