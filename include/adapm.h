@@ -35,9 +35,9 @@
  *     (the replicas of that call are not created and reads of those keys go
  *     to the main copy), ADAPM_ESTATE for a refcount overflow (more than
  *     65535 overlapping intents of one worker on one key).  ADAPM_ETIMEOUT
- *     reports that a bounded device-side wait gave up: the sort of keys runs
- *     as one cooperative launch whose blocks meet at grid barriers, and a
- *     barrier wait is limited.  Work enqueued after such a failure does not
+ *     reports that a bounded device-side wait gave up: the key sort of a
+ *     push runs as one cooperative launch whose blocks meet at grid
+ *     barriers, and a barrier wait is limited.  Work enqueued after such a failure does not
  *     touch the store, and the context is unusable afterwards (destroy it).
  *   - ADAPM_ECUDA reports a CUDA runtime error; the context is then unusable.
  *   - No C++ exception crosses the ABI.  A context is driven by one host
@@ -89,8 +89,8 @@ adapm_status adapm_destroy(adapm_ctx* ctx);
  * clock_start) or an expired one (clock_end <= C^worker) is a no-op.  A
  * window that contains the current clock is active at once: missing
  * replicas are created before the call's work ends.  Otherwise the keys are
- * sorted, de-duplicated and stored until the worker's clock reaches
- * clock_start.  Overlapping intents are reference-counted per (worker, key). */
+ * de-duplicated and stored until the worker's clock reaches clock_start.
+ * Overlapping intents are reference-counted per (worker, key). */
 adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                           int64_t clock_start, int64_t clock_end);
 

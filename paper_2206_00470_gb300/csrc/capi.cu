@@ -30,7 +30,7 @@ void adapm::note_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_orde
 namespace {
 
 struct IntentList {
-  uint32_t* keys = nullptr;   // device: cap sorted unique keys, then the count word
+  uint32_t* keys = nullptr;   // device: cap distinct keys (no particular order), then the count word
   uint32_t* count = nullptr;
   uint64_t cap = 0;
 };
@@ -59,6 +59,7 @@ struct adapm_ctx {
   std::string err;
   bool broken = false;
   unsigned long long bar_base = 0;   // dstate->bar_arrivals once the queued sorts have run
+  uint32_t intent_tag = 0;           // tag of the last Intent call (stamp array)
   uint64_t push_rows_host = 0;
   bool prof = false;
   std::vector<std::tuple<int, cudaEvent_t, cudaEvent_t>> pending;
@@ -233,8 +234,8 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &vb, n));
   CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
   uint32_t *sk = nullptr, *sp = nullptr;
-  CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, nullptr, nullptr,
-               ctx->sms, ctx->dstate, &ctx->bar_base, ctx->stream, &sk, &sp));
+  CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
+               &ctx->bar_base, ctx->stream, &sk, &sp));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
   float *ph = nullptr, *pt = nullptr;
@@ -334,7 +335,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       !dmalloc((void**)&s.acc, S * D * 4) || !dmalloc((void**)&s.map, W * K * 4) ||
       !dmalloc((void**)&s.rc, W * K * 2) || !dmalloc((void**)&s.holders, K * 4) ||
       !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
-      !dmalloc((void**)&s.ev_delta, K * 4) || !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
+      !dmalloc((void**)&s.ev_delta, K * 4) || !dmalloc((void**)&s.stamp, K * 4) ||
+      !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
     cudaGetLastError();
     return bail(ADAPM_ENOMEM);
   }
@@ -350,6 +352,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   ok &= cudaMemsetAsync(s.rc, 0, W * K * 2, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.holders, 0, K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.ev_delta, 0, K * 4, st) == cudaSuccess;
+  ok &= cudaMemsetAsync(s.stamp, 0, K * 4, st) == cudaSuccess;   // intent tags start at 1
   DevState h{};
   h.free_top = (int32_t)S;
   ok &= cudaMemcpyAsync(ctx->dstate, &h, sizeof h, cudaMemcpyHostToDevice, st) == cudaSuccess;
@@ -368,7 +371,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
-                  s.ev_delta, ctx->dstate};
+                  s.ev_delta, s.stamp, ctx->dstate};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& t : ctx->pending) {
@@ -401,16 +404,13 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   } else {
     Input<uint32_t> in;
     CK(stage_in(ctx, keys, n, &in));
-    uint32_t *ka = nullptr, *kb = nullptr, *hist = nullptr;
-    CK(pool_alloc(ctx, &ka, n));
-    CK(pool_alloc(ctx, &kb, n));
-    CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
-    CK(sort_keys(in.dev, n, ctx->s.K, false, ctx->bits, ka, kb, nullptr, nullptr, hist, L.keys, L.count,
-                 ctx->sms, ctx->dstate, &ctx->bar_base, ctx->stream, nullptr, nullptr));
+    if (++ctx->intent_tag == 0) {   // tags wrapped: clear the stamps
+      CK(cudaMemsetAsync(ctx->s.stamp, 0, ctx->s.K * 4, ctx->stream));
+      ctx->intent_tag = 1;
+    }
+    CK(cudaMemsetAsync(L.count, 0, sizeof(uint32_t), ctx->stream));
+    launch_intent_dedup(ctx->s, in.dev, n, ctx->intent_tag, L.keys, L.count, ctx->sms, ctx->stream);
     pool_free(ctx, in.owned);
-    pool_free(ctx, ka);
-    pool_free(ctx, kb);
-    pool_free(ctx, hist);
   }
   const int64_t id = ctx->next_list++;
   ctx->lists[id] = L;

@@ -9,6 +9,7 @@
 //   slot_owner  [S]    uint64   (w << 32) | k of a live slot, kEmptySlot if free
 //   free_stack  [S]    int32    free slots, top at free_stack[free_top - 1]
 //   ev_delta    [K]    int32    scratch for net refcount changes, kept zero
+//   stamp       [K]    uint32   tag of the last Intent call that listed k
 //   DevState                    counters and the sticky error bits
 #pragma once
 
@@ -64,6 +65,7 @@ struct Store {
   unsigned long long* slot_owner;
   int32_t* free_stack;
   int32_t* ev_delta;
+  uint32_t* stamp;
   DevState* st;
   uint64_t K;
   uint64_t S;
@@ -85,21 +87,18 @@ __device__ __forceinline__ bool sort_failed(const DevState* st) {
 // Stable sort of n uint32 keys by their low `bits` bits in one cooperative
 // launch on `stream`.  `raw` (n keys, not modified) is the first pass's
 // input; a key >= K is sorted as kNoKey (after every valid key) and sets
-// ERR_KEY_RANGE unless allow_nokey and it equals kNoKey.
-// ka/kb are ping-pong space of n keys; with va/vb non-null the positions
-// 0..n-1 travel with the keys.  The sorted keys (and positions) end in the
-// buffers returned through *keys_out / *pos_out.  If uniq_out is non-null,
-// the distinct keys other than kNoKey are written to it ascending and their
-// number to *uniq_count (0 if the sort gave up).  `scratch` holds
+// ERR_KEY_RANGE unless allow_nokey and it equals kNoKey.  ka/kb are
+// ping-pong space of n keys; with va/vb non-null the positions 0..n-1
+// travel with the keys.  The sorted keys (and positions) end in the buffers
+// returned through *keys_out / *pos_out.  `scratch` holds
 // sort_scratch_words(n) uint32 words.  *bar_base is the host's copy of
 // st->bar_arrivals, advanced by the launch.  If a grid-barrier wait gives
 // up, the kernel sets ERR_TIMEOUT and returns; every kernel that consumes a
 // sort checks that bit first and does nothing while it is set.
 size_t sort_scratch_words(uint64_t n);
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
-                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch,
-                      uint32_t* uniq_out, uint32_t* uniq_count, int sms, DevState* st,
-                      unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
+                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
+                      DevState* st, unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
                       uint32_t** pos_out);
 
 // Stream compaction (a count / scan / write pass), tmp of compact_tmp_words(n).

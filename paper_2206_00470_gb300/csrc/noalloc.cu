@@ -143,8 +143,8 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
   }
   ctx_add_push_rows(ctx, n);
   uint32_t *sk = nullptr, *sp = nullptr;
-  e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist),
-                nullptr, nullptr, v.sms, v.dstate, v.bar_base, v.stream, &sk, &sp);
+  e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist), v.sms,
+                v.dstate, v.bar_base, v.stream, &sk, &sp);
   if (e != cudaSuccess) {
     ctx_set_error(ctx, cudaGetErrorString(e));
     return ADAPM_ECUDA;

@@ -1,7 +1,5 @@
-// Stable LSD radix sort of uint32 keys (optionally carrying their positions)
-// and stream compaction, for the intent table (sort + unique of the keys of
-// one Intent call, Sec. 3) and for push (grouping a batch's delta rows by
-// key).
+// Stable LSD radix sort of uint32 keys carrying their positions, for push
+// (grouping a batch's delta rows by key, App. B.1.2), and stream compaction.
 //
 // Only ceil(log2(K + 1)) key bits are sorted, in ceil(bits / 9) passes of at
 // most 9 bits (512 buckets): 27-bit keys (100M) take 3 passes.  The whole
@@ -21,8 +19,7 @@
 //              digit and chunk of a warp)
 // so a pass costs two grid barriers.  With one sub-tile per chunk
 // (n <= 2048 B) the first pass's ranks are kept in registers from the
-// count.  The optional unique pass (count the first key of every run,
-// barrier, block offsets, write) is one more phase of the same launch.
+// count.
 //
 // The grid barrier is a monotonic arrival counter in DevState: the host
 // knows how many barriers each launch passes and hands the next launch its
@@ -128,8 +125,6 @@ struct SortArgs {
   uint32_t* vb;
   uint32_t* table;        // kDigits x gridDim.x (digit-major)
   uint32_t* totals;       // kDigits
-  uint32_t* uniq_out;
-  uint32_t* uniq_count;
   DevState* st;
   unsigned long long bar_base;   // st->bar_arrivals when the launch starts
   int allow_nokey;
@@ -242,36 +237,16 @@ __device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin
   __syncthreads();
 }
 
-// Distinct keys (kNoKey dropped) of the sorted keys in [i, i + kCompactItems)
-// per thread, as flags.
-__device__ __forceinline__ uint32_t first_of_run_flags(const uint32_t* keys, uint64_t i0, uint64_t end,
-                                                       bool (&f)[kCompactItems]) {
-  uint32_t c = 0;
-  uint32_t prev = i0 > 0 && i0 < end ? __ldcg(keys + i0 - 1) : kNoKey;
-#pragma unroll
-  for (int j = 0; j < kCompactItems; ++j) {
-    const uint64_t i = i0 + j;
-    const uint32_t k = i < end ? __ldcg(keys + i) : kNoKey;
-    f[j] = i < end && k != kNoKey && (i == 0 || k != prev);
-    prev = k;
-    c += f[j] ? 1u : 0u;
-  }
-  return c;
-}
-
 // Number of grid barriers one sort_kernel launch passes.
-__host__ __device__ constexpr uint32_t sort_barriers(int passes, bool uniq) {
-  return 2u * (uint32_t)passes + (uniq ? 2u : 0u);
-}
+__host__ __device__ constexpr uint32_t sort_barriers(int passes) { return 2u * (uint32_t)passes; }
 
-template <bool POS, bool UNIQ>
+template <bool POS>
 __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   __shared__ SortSmem sm;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const uint32_t B = gridDim.x;
   const uint32_t b = blockIdx.x;
-  if (UNIQ && b == 0 && threadIdx.x == 0) *a.uniq_count = 0;
   // an earlier sort gave up: the barrier state is unknown, so do nothing
   if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
   __syncthreads();
@@ -490,7 +465,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
       }
       __syncthreads();
     }
-    if (more || UNIQ) {
+    if (more) {
       if (!grid_barrier(a, nbar, sm)) return;
     }
     kin = kout;
@@ -499,40 +474,6 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     vout = vout == a.va ? a.vb : a.va;
     shift = nshift;
   }
-  if (!UNIQ) return;
-  // unique: count, barrier, block offset, write
-  uint32_t cnt = 0;
-  for (uint64_t s0 = c0; s0 < c1; s0 += kTile) {
-    bool f[kCompactItems];
-    const uint64_t s1 = s0 + kTile < c1 ? s0 + kTile : c1;
-    cnt += first_of_run_flags(kin, s0 + (uint64_t)threadIdx.x * kCompactItems, s1, f);
-  }
-  {
-    uint32_t total;
-    block_exclusive_scan<kSortThreads>(cnt, &total, sm.scan);
-    if (threadIdx.x == 0) a.table[b] = total;
-  }
-  if (!grid_barrier(a, nbar, sm)) return;
-  uint32_t before = 0;
-  for (uint32_t j = threadIdx.x; j < b; j += kSortThreads) before += __ldcg(a.table + j);
-  {
-    uint32_t total;
-    block_exclusive_scan<kSortThreads>(before, &total, sm.scan);
-    before = total;
-  }
-  for (uint64_t s0 = c0; s0 < c1; s0 += kTile) {
-    bool f[kCompactItems];
-    const uint64_t s1 = s0 + kTile < c1 ? s0 + kTile : c1;
-    const uint64_t i0 = s0 + (uint64_t)threadIdx.x * kCompactItems;
-    const uint32_t c = first_of_run_flags(kin, i0, s1, f);
-    uint32_t total;
-    uint32_t pos = before + block_exclusive_scan<kSortThreads>(c, &total, sm.scan);
-#pragma unroll
-    for (int j = 0; j < kCompactItems; ++j)
-      if (f[j]) a.uniq_out[pos++] = __ldcg(kin + i0 + j);
-    before += total;
-  }
-  if (b == B - 1 && threadIdx.x == 0) *a.uniq_count = before;
 }
 
 // ---- compaction ------------------------------------------------------------
@@ -610,11 +551,11 @@ void compact(Sel sel, uint32_t* out, uint32_t* count, uint32_t* tmp, cudaStream_
 
 // Resident blocks per SM of one sort_kernel instance (its shared memory and
 // registers), looked up once.
-template <bool POS, bool UNIQ>
+template <bool POS>
 int sort_blocks_per_sm() {
   static const int occ = [] {
     int o = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS, UNIQ>, kSortThreads, 0) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS>, kSortThreads, 0) !=
         cudaSuccess) {
       cudaGetLastError();
       o = 1;
@@ -624,9 +565,9 @@ int sort_blocks_per_sm() {
   return occ;
 }
 
-template <bool POS, bool UNIQ>
+template <bool POS>
 cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cudaStream_t stream) {
-  const int occ = sort_blocks_per_sm<POS, UNIQ>();
+  const int occ = sort_blocks_per_sm<POS>();
   uint64_t B = (a.n + kSub - 1) / kSub;
   const uint64_t resident = (uint64_t)sms * (occ < 4 ? occ : 4);
   if (B > resident) B = resident;
@@ -635,9 +576,9 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   a.bar_base = *bar_base;
   void* params[] = {&a};
   note_launches(1);
-  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, UNIQ>, dim3((unsigned)B),
+  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS>, dim3((unsigned)B),
                                                     dim3(kSortThreads), params, 0, stream);
-  if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes, UNIQ) * B;
+  if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes) * B;
   return e;
 }
 
@@ -657,17 +598,13 @@ size_t sort_scratch_words(uint64_t n) {
 }
 
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
-                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch,
-                      uint32_t* uniq_out, uint32_t* uniq_count, int sms, DevState* st,
-                      unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
+                      uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
+                      DevState* st, unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
                       uint32_t** pos_out) {
   const PassPlan pl = plan_for(bits);
   if (keys_out) *keys_out = pl.passes % 2 ? ka : kb;
   if (pos_out) *pos_out = va ? (pl.passes % 2 ? va : vb) : nullptr;
-  if (n == 0) {
-    if (uniq_count) return cudaMemsetAsync(uniq_count, 0, sizeof(uint32_t), stream);
-    return cudaSuccess;
-  }
+  if (n == 0) return cudaSuccess;
   SortArgs a;
   a.raw = raw;
   a.n = n;
@@ -678,19 +615,13 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
   a.vb = vb;
   a.totals = scratch + kScratchHead;
   a.table = scratch + kScratchHead + kDigits;
-  a.uniq_out = uniq_out;
-  a.uniq_count = uniq_count;
   a.st = st;
   a.allow_nokey = allow_nokey ? 1 : 0;
   a.passes = pl.passes;
   a.per = pl.per;
   a.bits = bits;
-  const bool pos = va != nullptr;
-  const bool uniq = uniq_out != nullptr;
-  if (pos && uniq) return launch_sort<true, true>(a, bar_base, sms, stream);
-  if (pos) return launch_sort<true, false>(a, bar_base, sms, stream);
-  if (uniq) return launch_sort<false, true>(a, bar_base, sms, stream);
-  return launch_sort<false, false>(a, bar_base, sms, stream);
+  if (va) return launch_sort<true>(a, bar_base, sms, stream);
+  return launch_sort<false>(a, bar_base, sms, stream);
 }
 
 size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile + 1); }

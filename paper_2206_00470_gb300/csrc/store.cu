@@ -61,6 +61,50 @@ __device__ __forceinline__ void block_sum2(uint32_t& a, uint32_t& b) {
   }
 }
 
+// Exclusive block-wide scans of two per-thread counts (every thread of the
+// block calls it); ta / tb receive the block totals.
+__device__ __forceinline__ void block_exclusive_scan2(uint32_t& a, uint32_t& b, uint32_t& ta, uint32_t& tb) {
+  __shared__ uint32_t sa[32], sb[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  uint32_t xa = a, xb = b;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, xa, o);
+    const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, xb, o);
+    if (lane >= o) {
+      xa += ya;
+      xb += yb;
+    }
+  }
+  if (lane == 31) {
+    sa[warp] = xa;
+    sb[warp] = xb;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    uint32_t va = lane < nw ? sa[lane] : 0u, vb = lane < nw ? sb[lane] : 0u;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, va, o);
+      const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, vb, o);
+      if (lane >= o) {
+        va += ya;
+        vb += yb;
+      }
+    }
+    if (lane < nw) {
+      sa[lane] = va;
+      sb[lane] = vb;
+    }
+  }
+  __syncthreads();
+  a = (warp > 0 ? sa[warp - 1] : 0u) + xa - a;
+  b = (warp > 0 ? sb[warp - 1] : 0u) + xb - b;
+  ta = sa[nw - 1];
+  tb = sb[nw - 1];
+  __syncthreads();
+}
+
 template <int G>
 __device__ __forceinline__ uint64_t group_id() {
   return ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) / G;
@@ -541,6 +585,72 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
 }
 
 // ---------------------------------------------------------------------------
+// intent: the distinct keys of one call (Sec. 3: an intent names a set of
+// parameters, so a key listed twice in one call counts once)
+// ---------------------------------------------------------------------------
+constexpr int kDedupItems = 8;
+constexpr int kDedupTile = kThreads * kDedupItems;   // keys per block and round
+constexpr int kDedupTab = 2 * kDedupTile;            // shared hash table, half full at most
+
+// Each block takes tiles of 2048 keys: a shared-memory hash set (open
+// addressing) keeps the first copy of every key of the tile, and an exchange
+// on the key's stamp keeps the first copy over all tiles (stamp == tag once
+// some copy has been listed).  One atomic per block and round appends.
+__global__ void __launch_bounds__(kThreads) intent_dedup_kernel(Store s, const uint32_t* __restrict__ keys,
+                                                                uint64_t n, uint32_t tag,
+                                                                uint32_t* __restrict__ out, uint32_t* count) {
+  __shared__ uint32_t tab[kDedupTab];
+  __shared__ uint32_t base_s;
+  bool bad = false;
+  for (uint64_t t0 = (uint64_t)blockIdx.x * kDedupTile; t0 < n;
+       t0 += (uint64_t)gridDim.x * kDedupTile) {   // block-uniform trip count
+    for (int i = threadIdx.x; i < kDedupTab; i += kThreads) tab[i] = kNoKey;
+    __syncthreads();
+    uint32_t k[kDedupItems];
+    bool first[kDedupItems];
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) {
+      const uint64_t i = t0 + (uint64_t)it * kThreads + threadIdx.x;
+      k[it] = i < n ? __ldg(keys + i) : kNoKey;
+      if (i < n && k[it] >= s.K) {
+        bad = true;
+        k[it] = kNoKey;
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) {
+      first[it] = false;
+      if (k[it] == kNoKey) continue;
+      uint32_t h = (k[it] * 0x9E3779B1u) >> (32 - 12);   // 12 bits: kDedupTab = 4096
+      for (int probe = 0; probe < kDedupTab; ++probe) {
+        const uint32_t old = atomicCAS(&tab[h], kNoKey, k[it]);
+        if (old == kNoKey) {
+          first[it] = true;
+          break;
+        }
+        if (old == k[it]) break;
+        h = (h + 1) & (kDedupTab - 1);
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it)
+      if (first[it]) first[it] = atomicExch(s.stamp + k[it], tag) != tag;
+    uint32_t c = 0, unused = 0, total, t2;
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) c += first[it] ? 1u : 0u;
+    block_exclusive_scan2(c, unused, total, t2);
+    if (threadIdx.x == 0) base_s = total ? atomicAdd(count, total) : 0u;
+    __syncthreads();
+    c += base_s;
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it)
+      if (first[it]) out[c++] = k[it];
+    __syncthreads();
+  }
+  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(s.st, ERR_KEY_RANGE);
+}
+
+// ---------------------------------------------------------------------------
 // intent events -> refcounts -> create / evict lists
 // ---------------------------------------------------------------------------
 // Up to kEventLists intent lists handled by one launch.
@@ -567,50 +677,6 @@ __global__ void events_add_kernel(EventBatch eb, int32_t* __restrict__ ev_delta,
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
       atomicAdd(ev_delta + keys[i], eb.sign[l]);
   }
-}
-
-// Exclusive block-wide scans of two per-thread counts (every thread of the
-// block calls it); ta / tb receive the block totals.
-__device__ __forceinline__ void block_exclusive_scan2(uint32_t& a, uint32_t& b, uint32_t& ta, uint32_t& tb) {
-  __shared__ uint32_t sa[32], sb[32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-  uint32_t xa = a, xb = b;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, xa, o);
-    const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, xb, o);
-    if (lane >= o) {
-      xa += ya;
-      xb += yb;
-    }
-  }
-  if (lane == 31) {
-    sa[warp] = xa;
-    sb[warp] = xb;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    uint32_t va = lane < nw ? sa[lane] : 0u, vb = lane < nw ? sb[lane] : 0u;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t ya = __shfl_up_sync(0xFFFFFFFFu, va, o);
-      const uint32_t yb = __shfl_up_sync(0xFFFFFFFFu, vb, o);
-      if (lane >= o) {
-        va += ya;
-        vb += yb;
-      }
-    }
-    if (lane < nw) {
-      sa[lane] = va;
-      sb[lane] = vb;
-    }
-  }
-  __syncthreads();
-  a = (warp > 0 ? sa[warp - 1] : 0u) + xa - a;
-  b = (warp > 0 ? sb[warp - 1] : 0u) + xb - b;
-  ta = sa[nw - 1];
-  tb = sb[nw - 1];
-  __syncthreads();
 }
 
 // Net refcount change of every listed key (4 keys per thread per round, each
@@ -1026,6 +1092,15 @@ unsigned grid_for(uint64_t groups, int G, int sms) {
 // ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
+void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint32_t tag, uint32_t* out,
+                         uint32_t* count, int sms, cudaStream_t stream) {
+  if (n == 0) return;
+  uint64_t b = (n + kDedupTile - 1) / kDedupTile;
+  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+  note_launches(1);
+  intent_dedup_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, keys, n, tag, out, count);
+}
+
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream) {
   if (n == 0) return;

@@ -30,7 +30,7 @@ uint64_t push_long_part_rows(uint64_t nchunks);
 // Rows per push chunk for value length D and a batch of n rows.
 uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms);
 
-// One stored intent list (sorted unique keys, device count) and the sign of
+// One stored intent list (distinct keys, device count) and the sign of
 // its refcount event: +1 when its window opens, -1 when it closes.
 struct EventList {
   const uint32_t* keys;
@@ -39,6 +39,12 @@ struct EventList {
   int sign;
 };
 
+// The distinct keys of one Intent call (keys >= K set ERR_KEY_RANGE and are
+// dropped), in no particular order, appended to out; *count (zeroed by the
+// caller) receives their number.  `tag` must differ from every stamp left
+// by earlier calls.
+void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint32_t tag, uint32_t* out,
+                         uint32_t* count, int sms, cudaStream_t stream);
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream);
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream);
