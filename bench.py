@@ -42,25 +42,30 @@ from synth import workloads as wl  # noqa: E402
 
 METRIC = "pulled+pushed keys/s and training samples/s on 1 GB300; % of HBM roofline"
 
-# DRAM bytes (read + write) of the push scatter kernels per pushed row of the MF workload, from the
-# capture summarised in profiles/push_scatter_mf_2Mx200K.md (79.1 MB per 65,536-row push); it stands for
-# the kernels only while their source is the one captured (first 16 hex digits of its sha256).
-PUSH_TRAFFIC = {"workload": "mf", "bytes_per_row": 79.1e6 / 65536,
-                "source": "paper_2206_00470_gb300/csrc/store.cu", "sha256_16": "6c51440c2c90c933"}
+# DRAM bytes (read + write) of the push scatter kernels (push_chunks + push_fixup + push_long) per
+# pushed row, per workload, from the full ncu captures summarised in profiles/ (each on a smaller case
+# of the same workload, scaled by rows); a figure stands for the kernels only while their source is the
+# one captured (first 16 hex digits of its sha256), otherwise the traffic is reported as null.
+PUSH_SOURCE = "paper_2206_00470_gb300/csrc/store.cu"
+PUSH_TRAFFIC = {
+    "mf": {"bytes_per_row": 80.1e6 / 65536, "sha256_16": "394a24f7083becd6"},   # profiles/push_scatter_mf_2Mx200K.md
+    "micro": {"bytes_per_row": None, "sha256_16": None},
+}
 
 
 def recorded_traffic(workload, rows_per_launch):
     import hashlib
-    if workload != PUSH_TRAFFIC["workload"]:
+    rec = PUSH_TRAFFIC.get(workload)
+    if not rec or rec["bytes_per_row"] is None:
         return None
     try:
-        with open(os.path.join(ROOT, PUSH_TRAFFIC["source"]), "rb") as f:
+        with open(os.path.join(ROOT, PUSH_SOURCE), "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()[:16]
     except OSError:
         return None
-    if sha != PUSH_TRAFFIC["sha256_16"]:
+    if sha != rec["sha256_16"]:
         return None
-    return PUSH_TRAFFIC["bytes_per_row"] * rows_per_launch
+    return rec["bytes_per_row"] * rows_per_launch
 UNIT = "keys/s"
 
 
