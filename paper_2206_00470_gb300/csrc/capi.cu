@@ -233,9 +233,6 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &va, n));
   CK(pool_alloc(ctx, &vb, n));
   CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
-  uint32_t *sk = nullptr, *sp = nullptr;
-  CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
-               &ctx->bar_base, ctx->stream, &sk, &sp));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
   float *ph = nullptr, *pt = nullptr;
@@ -245,8 +242,10 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   float* lparts = nullptr;
   CK(pool_alloc(ctx, &longs, push_long_list_words(nchunks)));
   CK(pool_alloc(ctx, &lparts, push_long_part_rows(nchunks) * ctx->s.D));
-  CK(cudaMemsetAsync(longs, 0, sizeof(uint32_t), ctx->stream));
-  CK(cudaMemsetAsync(&ctx->dstate->last_unique, 0, sizeof(uint32_t), ctx->stream));
+  // the sort also clears the hot-key list count and the distinct-key counter
+  uint32_t *sk = nullptr, *sp = nullptr;
+  CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
+               &ctx->bar_base, longs, &ctx->dstate->last_unique, ctx->stream, &sk, &sp));
   ctx->push_rows_host += n;
   PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, longs + 1, longs, lparts};
   {

@@ -92,14 +92,16 @@ __device__ __forceinline__ bool sort_failed(const DevState* st) {
 // travel with the keys.  The sorted keys (and positions) end in the buffers
 // returned through *keys_out / *pos_out.  `scratch` holds
 // sort_scratch_words(n) uint32 words.  *bar_base is the host's copy of
-// st->bar_arrivals, advanced by the launch.  If a grid-barrier wait gives
+// st->bar_arrivals, advanced by the launch.  clear0 / clear1 (may be null)
+// are device words the launch sets to zero before any later kernel on the
+// stream runs (counters of the consumer).  If a grid-barrier wait gives
 // up, the kernel sets ERR_TIMEOUT and returns; every kernel that consumes a
 // sort checks that bit first and does nothing while it is set.
 size_t sort_scratch_words(uint64_t n);
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
-                      DevState* st, unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
-                      uint32_t** pos_out);
+                      DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
+                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out);
 
 // Stream compaction (a count / scan / write pass), tmp of compact_tmp_words(n).
 size_t compact_tmp_words(uint64_t n);

@@ -135,16 +135,12 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
   }
   auto at = [&](size_t off) { return reinterpret_cast<uint32_t*>(base + off); };
   uint32_t* longs = at(L.longs);
-  // the array keeps the previous call's contents: zero the hot-key list count
-  if (cudaMemsetAsync(longs, 0, sizeof(uint32_t), v.stream) != cudaSuccess ||
-      cudaMemsetAsync(&v.dstate->last_unique, 0, sizeof(uint32_t), v.stream) != cudaSuccess) {
-    ctx_set_error(ctx, "cudaMemsetAsync failed");
-    return ADAPM_ECUDA;
-  }
   ctx_add_push_rows(ctx, n);
   uint32_t *sk = nullptr, *sp = nullptr;
+  // the array keeps the previous call's contents: the sort clears the
+  // hot-key list count (and the distinct-key counter)
   e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist), v.sms,
-                v.dstate, v.bar_base, v.stream, &sk, &sp);
+                v.dstate, v.bar_base, longs, &v.dstate->last_unique, v.stream, &sk, &sp);
   if (e != cudaSuccess) {
     ctx_set_error(ctx, cudaGetErrorString(e));
     return ADAPM_ECUDA;

@@ -126,6 +126,8 @@ struct SortArgs {
   uint32_t* table;        // kDigits x gridDim.x (digit-major)
   uint32_t* totals;       // kDigits
   DevState* st;
+  uint32_t* clear0;              // words set to zero by the launch (nullptr: none)
+  uint32_t* clear1;
   unsigned long long bar_base;   // st->bar_arrivals when the launch starts
   int allow_nokey;
   int passes;
@@ -247,6 +249,10 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   const int warp = threadIdx.x >> 5;
   const uint32_t B = gridDim.x;
   const uint32_t b = blockIdx.x;
+  if (b == 0 && threadIdx.x == 0) {
+    if (a.clear0) *a.clear0 = 0u;
+    if (a.clear1) *a.clear1 = 0u;
+  }
   // an earlier sort gave up: the barrier state is unknown, so do nothing
   if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
   __syncthreads();
@@ -599,8 +605,8 @@ size_t sort_scratch_words(uint64_t n) {
 
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
-                      DevState* st, unsigned long long* bar_base, cudaStream_t stream, uint32_t** keys_out,
-                      uint32_t** pos_out) {
+                      DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
+                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out) {
   const PassPlan pl = plan_for(bits);
   if (keys_out) *keys_out = pl.passes % 2 ? ka : kb;
   if (pos_out) *pos_out = va ? (pl.passes % 2 ? va : vb) : nullptr;
@@ -616,6 +622,8 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
   a.totals = scratch + kScratchHead;
   a.table = scratch + kScratchHead + kDigits;
   a.st = st;
+  a.clear0 = clear0;
+  a.clear1 = clear1;
   a.allow_nokey = allow_nokey ? 1 : 0;
   a.passes = pl.passes;
   a.per = pl.per;

@@ -679,10 +679,9 @@ __global__ void events_add_kernel(EventBatch eb, int32_t* __restrict__ ev_delta,
   }
 }
 
-// Net refcount change of every listed key (4 keys per thread per round, each
-// step a round of independent accesses), appended to the create list (0 ->
-// >0) or the evict list (>0 -> 0, if a replica exists).  The order of a list
-// is not specified.
+// Net refcount change of every listed key (4 keys per thread per round),
+// appended to the create list (0 -> >0) or the evict list (>0 -> 0, if a
+// replica exists).  The order of a list is not specified.
 __global__ void events_apply_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* create_list,
                                     uint32_t* evict_list) {
   if (sort_failed(s.st)) return;
