@@ -34,8 +34,9 @@ namespace {
 
 constexpr int kSortThreads = 256;
 constexpr int kWarps = kSortThreads / 32;
-constexpr int kItems = 8;                          // keys per thread per sub-tile
-constexpr int kSub = kSortThreads * kItems;        // 2048 keys per sub-tile
+constexpr int kItems = 8;                          // keys per thread per sub-tile (largest)
+constexpr int kSub = kSortThreads * kItems;        // 2048 keys per sub-tile (largest)
+constexpr int kSubMin = kSortThreads * 4;          // sub-tile of small batches (4 keys per thread)
 constexpr int kRadixBits = 9;
 constexpr int kDigits = 1 << kRadixBits;           // 512
 constexpr int kDPT = kDigits / kSortThreads;       // digits per thread (2)
@@ -181,17 +182,17 @@ __device__ bool grid_barrier(const SortArgs& a, uint32_t& nbar, SortSmem& sm) {
 // of digit d in the sub-tile, rank[it] = earlier keys of the same digit in
 // the same warp.  `first`: keys come from the caller's array (mapped to
 // kNoKey when out of range, positions are the indices).
-template <bool POS>
+template <bool POS, int ITEMS>
 __device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin, const uint32_t* vin,
                                           bool first, uint64_t s0, uint64_t s1, int shift, int nbits,
-                                          uint32_t (&key)[kItems], uint32_t (&val)[kItems],
-                                          uint32_t (&rank)[kItems], bool& bad, SortSmem& sm) {
+                                          uint32_t (&key)[ITEMS], uint32_t (&val)[ITEMS],
+                                          uint32_t (&rank)[ITEMS], bool& bad, SortSmem& sm) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   for (int i = threadIdx.x; i < kWarps * kDigits; i += kSortThreads) (&sm.wcnt[0][0])[i] = 0;
 #pragma unroll
-  for (int it = 0; it < kItems; ++it) {
-    const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+  for (int it = 0; it < ITEMS; ++it) {
+    const uint64_t i = s0 + ((uint64_t)(warp * ITEMS + it) << 5) + lane;
     const bool valid = i < s1;
     uint32_t k = 0;
     if (valid) {
@@ -212,8 +213,8 @@ __device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin
   const uint32_t mask = (1u << nbits) - 1u;
   const uint32_t lt = lanemask_lt();
 #pragma unroll
-  for (int it = 0; it < kItems; ++it) {
-    const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+  for (int it = 0; it < ITEMS; ++it) {
+    const uint64_t i = s0 + ((uint64_t)(warp * ITEMS + it) << 5) + lane;
     const bool valid = i < s1;
     const uint32_t d = (key[it] >> shift) & mask;
     const uint32_t peers = digit_peers(d, valid, nbits);
@@ -242,8 +243,9 @@ __device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin
 // Number of grid barriers one sort_kernel launch passes.
 __host__ __device__ constexpr uint32_t sort_barriers(int passes) { return 2u * (uint32_t)passes; }
 
-template <bool POS>
+template <bool POS, int ITEMS>
 __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
+  constexpr int SUB = kSortThreads * ITEMS;   // keys per sub-tile
   __shared__ SortSmem sm;
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -261,21 +263,21 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   const uint64_t chunk = (a.n + B - 1) / B;
   const uint64_t c0 = a.n < b * chunk ? a.n : b * chunk;
   const uint64_t c1 = a.n < c0 + chunk ? a.n : c0 + chunk;
-  const bool single = c1 - c0 <= (uint64_t)kSub;
+  const bool single = c1 - c0 <= (uint64_t)SUB;
   uint32_t* const table0 = a.table;                       // passes 0, 2, ...
   uint32_t* const table1 = a.table + (uint64_t)kDigits * B;   // passes 1, 3, ...
   const uint32_t* kin = a.raw;
   const uint32_t* vin = nullptr;
   uint32_t* kout = a.ka;
   uint32_t* vout = a.va;
-  uint32_t key[kItems], val[kItems], rank[kItems];
+  uint32_t key[ITEMS], val[ITEMS], rank[ITEMS];
   bool bad = false;
   // 0. first pass digit counts of the chunk (ranks kept when one sub-tile)
   {
     const int nbits = a.per < a.bits ? a.per : a.bits;
     const uint32_t mask = (1u << nbits) - 1u;
     if (single) {
-      load_rank<POS>(a, kin, vin, true, c0, c1, 0, nbits, key, val, rank, bad, sm);
+      load_rank<POS, ITEMS>(a, kin, vin, true, c0, c1, 0, nbits, key, val, rank, bad, sm);
     } else {
       for (int d = threadIdx.x; d < kDigits; d += kSortThreads) sm.cnt[d] = 0;
       __syncthreads();
@@ -416,9 +418,10 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
         run += v[q];
       }
     }
-    for (uint64_t s0 = c0; s0 < c1; s0 += kSub) {
-      const uint64_t s1 = s0 + kSub < c1 ? s0 + kSub : c1;
-      if (!(single && first)) load_rank<POS>(a, kin, vin, first, s0, s1, shift, nbits, key, val, rank, bad, sm);
+    for (uint64_t s0 = c0; s0 < c1; s0 += SUB) {
+      const uint64_t s1 = s0 + SUB < c1 ? s0 + SUB : c1;
+      if (!(single && first))
+        load_rank<POS, ITEMS>(a, kin, vin, first, s0, s1, shift, nbits, key, val, rank, bad, sm);
       {
         uint32_t local = 0;
 #pragma unroll
@@ -434,8 +437,8 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
       }
       __syncthreads();
 #pragma unroll
-      for (int it = 0; it < kItems; ++it) {
-        const uint64_t i = s0 + ((uint64_t)(warp * kItems + it) << 5) + lane;
+      for (int it = 0; it < ITEMS; ++it) {
+        const uint64_t i = s0 + ((uint64_t)(warp * ITEMS + it) << 5) + lane;
         if (i < s1) {
           const uint32_t d = (key[it] >> shift) & mask;
           const uint32_t lp = sm.lofs[d] + sm.wcnt[warp][d] + rank[it];
@@ -557,11 +560,11 @@ void compact(Sel sel, uint32_t* out, uint32_t* count, uint32_t* tmp, cudaStream_
 
 // Resident blocks per SM of one sort_kernel instance (its shared memory and
 // registers), looked up once.
-template <bool POS>
+template <bool POS, int ITEMS>
 int sort_blocks_per_sm() {
   static const int occ = [] {
     int o = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS>, kSortThreads, 0) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS, ITEMS>, kSortThreads, 0) !=
         cudaSuccess) {
       cudaGetLastError();
       o = 1;
@@ -571,10 +574,11 @@ int sort_blocks_per_sm() {
   return occ;
 }
 
-template <bool POS>
+template <bool POS, int ITEMS>
 cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cudaStream_t stream) {
-  const int occ = sort_blocks_per_sm<POS>();
-  uint64_t B = (a.n + kSub - 1) / kSub;
+  constexpr uint64_t SUB = (uint64_t)kSortThreads * ITEMS;
+  const int occ = sort_blocks_per_sm<POS, ITEMS>();
+  uint64_t B = (a.n + SUB - 1) / SUB;
   const uint64_t resident = (uint64_t)sms * (occ < 4 ? occ : 4);
   if (B > resident) B = resident;
   if (B > kMaxSortBlocks) B = kMaxSortBlocks;
@@ -582,7 +586,7 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   a.bar_base = *bar_base;
   void* params[] = {&a};
   note_launches(1);
-  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS>, dim3((unsigned)B),
+  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, ITEMS>, dim3((unsigned)B),
                                                     dim3(kSortThreads), params, 0, stream);
   if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes) * B;
   return e;
@@ -597,7 +601,7 @@ int bits_for(uint64_t num_keys) {
 }
 
 size_t sort_scratch_words(uint64_t n) {
-  uint64_t rows = (n + kSub - 1) / kSub;
+  uint64_t rows = (n + kSubMin - 1) / kSubMin;
   if (rows > kMaxSortBlocks) rows = kMaxSortBlocks;
   if (rows < 1) rows = 1;
   return (size_t)(kScratchHead + kDigits + 2 * rows * kDigits);   // totals, two tables
@@ -628,8 +632,11 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
   a.passes = pl.passes;
   a.per = pl.per;
   a.bits = bits;
-  if (va) return launch_sort<true>(a, bar_base, sms, stream);
-  return launch_sort<false>(a, bar_base, sms, stream);
+  // batches that would give fewer blocks than SMs take sub-tiles of half the
+  // size: twice the blocks, half the ranking work per block
+  if ((n + kSub - 1) / kSub < (uint64_t)sms)
+    return va ? launch_sort<true, 4>(a, bar_base, sms, stream) : launch_sort<false, 4>(a, bar_base, sms, stream);
+  return va ? launch_sort<true, kItems>(a, bar_base, sms, stream) : launch_sort<false, kItems>(a, bar_base, sms, stream);
 }
 
 size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile + 1); }
