@@ -197,17 +197,19 @@ __device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, u
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   float4* main4 = reinterpret_cast<float4*>(s.main);
   float4* t1 = sl >= 0 ? val4 + (uint64_t)sl * D4 : main4 + (uint64_t)k * D4;
+  // the segment is the only writer of its targets: vector atomic adds give
+  // the plain fp32 sums without a round trip of the target rows
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const uint32_t col = lane + c * G;
-    if (col < D4) t1[col] = f4add(t1[col], sum[c]);
+    if (col < D4) atomicAdd(t1 + col, sum[c]);
   }
   if (sl >= 0) {
     float4* t2 = acc4 + (uint64_t)sl * D4;
 #pragma unroll
     for (int c = 0; c < C; ++c) {
       const uint32_t col = lane + c * G;
-      if (col < D4) t2[col] = f4add(t2[col], sum[c]);
+      if (col < D4) atomicAdd(t2 + col, sum[c]);
     }
   }
 }
@@ -289,11 +291,11 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
 #pragma unroll
     for (int c = 0; c < C; ++c) run[c] = f4zero();
     for (uint32_t p = p0; p < p1; p += R) {
-      // one round of loads: delta rows and the targets of whole segments ending here
+      // one round of loads: the delta rows
       uint8_t f[R];
       int32_t sl[R];
       uint32_t k[R];
-      float4 d[R][C], tv[R][C], ta[R][C];
+      float4 d[R][C];
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         const bool v = p + r < p1;
@@ -301,17 +303,13 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
         sl[r] = (f[r] & 7) == 7 ? ss[p + r] : -2;
         k[r] = v ? sk[1 + p + r] : kNoKey;
         const uint32_t src = v ? sp[p + r] : 0u;
-        const float4* tvp = sl[r] >= 0 ? val4 + (uint64_t)sl[r] * D4 : main4 + (uint64_t)k[r] * D4;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          const bool cv = col < D4;
-          d[r][c] = ((f[r] & 16) && cv) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
-          tv[r][c] = (sl[r] != -2 && cv) ? tvp[col] : f4zero();
-          ta[r][c] = (sl[r] >= 0 && cv) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
+          d[r][c] = ((f[r] & 16) && col < D4) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
         }
       }
-      // running sums in position order, then the stores
+      // running sums in position order
 #pragma unroll
       for (int r = 0; r < R; ++r) {
 #pragma unroll
@@ -320,6 +318,10 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
           d[r][c] = run[c];
         }
       }
+      // a whole segment's sum goes to its targets by vector atomic adds: the
+      // segment is the only writer of those rows in this kernel, so the
+      // result is the plain fp32 sum target + s, and no target row has to
+      // travel to the SM and back
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         if (sl[r] != -2) {
@@ -327,13 +329,13 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
 #pragma unroll
           for (int c = 0; c < C; ++c) {
             const uint32_t col = lane + c * G;
-            if (col < D4) dst[col] = f4add(tv[r][c], d[r][c]);
+            if (col < D4) atomicAdd(dst + col, d[r][c]);
           }
           if (sl[r] >= 0) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
               const uint32_t col = lane + c * G;
-              if (col < D4) acc4[(uint64_t)sl[r] * D4 + col] = f4add(ta[r][c], d[r][c]);
+              if (col < D4) atomicAdd(acc4 + (uint64_t)sl[r] * D4 + col, d[r][c]);
             }
           }
         } else if (f[r] & 1) {
