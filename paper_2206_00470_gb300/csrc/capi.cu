@@ -215,6 +215,7 @@ adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventLis
   uint32_t *create_list = nullptr, *evict_list = nullptr;
   CK(pool_alloc(ctx, &create_list, total));
   CK(pool_alloc(ctx, &evict_list, total));
+  CK(cudaMemsetAsync(&ctx->dstate->n_create, 0, 2 * sizeof(uint32_t), ctx->stream));
   launch_events(ctx->s, w, ev.data(), (int)ev.size(), create_list, evict_list, ctx->sms, ctx->stream);
   launch_evict_create(ctx->s, w, create_list, evict_list, total, ctx->sms, ctx->stream);
   pool_free(ctx, create_list);
@@ -332,9 +333,9 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   auto dmalloc = [&](void** p, size_t bytes) { return cudaMalloc(p, bytes) == cudaSuccess; };
   if (!dmalloc((void**)&s.main, K * D * 4) || !dmalloc((void**)&s.val, S * D * 4) ||
       !dmalloc((void**)&s.acc, S * D * 4) || !dmalloc((void**)&s.map, W * K * 4) ||
-      !dmalloc((void**)&s.rc, W * K * 2) || !dmalloc((void**)&s.holders, K * 4) ||
+      !dmalloc((void**)&s.rc, W * K * 4) || !dmalloc((void**)&s.holders, K * 4) ||
       !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
-      !dmalloc((void**)&s.ev_delta, K * 4) || !dmalloc((void**)&s.stamp, K * 4) ||
+      !dmalloc((void**)&s.stamp, K * 4) ||
       !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
     cudaGetLastError();
     return bail(ADAPM_ENOMEM);
@@ -348,9 +349,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
     ok &= cudaMemsetAsync(s.main, 0, K * D * 4, st) == cudaSuccess;
   }
   ok &= cudaMemsetAsync(s.map, 0xFF, W * K * 4, st) == cudaSuccess;   // -1: no replica
-  ok &= cudaMemsetAsync(s.rc, 0, W * K * 2, st) == cudaSuccess;
+  ok &= cudaMemsetAsync(s.rc, 0, W * K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.holders, 0, K * 4, st) == cudaSuccess;
-  ok &= cudaMemsetAsync(s.ev_delta, 0, K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.stamp, 0, K * 4, st) == cudaSuccess;   // intent tags start at 1
   DevState h{};
   h.free_top = (int32_t)S;
@@ -370,7 +370,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
-                  s.ev_delta, s.stamp, ctx->dstate};
+                  s.stamp, ctx->dstate};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& t : ctx->pending) {

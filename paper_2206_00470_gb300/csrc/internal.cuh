@@ -4,11 +4,10 @@
 //   main        [K][D] fp32     main copy of every parameter
 //   val, acc    [S][D] fp32     replica pool: local value and pending updates
 //   map         [W][K] int32    slot of worker w's replica of key k, or -1
-//   rc          [W][K] uint16   number of w's active intents containing k
+//   rc          [W][K] uint32   number of w's active intents containing k
 //   holders     [K]    uint32   bit w set iff worker w holds a replica of k
 //   slot_owner  [S]    uint64   (w << 32) | k of a live slot, kEmptySlot if free
 //   free_stack  [S]    int32    free slots, top at free_stack[free_top - 1]
-//   ev_delta    [K]    int32    scratch for net refcount changes, kept zero
 //   stamp       [K]    uint32   tag of the last Intent call that listed k
 //   DevState                    counters and the sticky error bits
 #pragma once
@@ -60,11 +59,10 @@ struct Store {
   float* val;
   float* acc;
   int32_t* map;
-  uint16_t* rc;
+  uint32_t* rc;
   uint32_t* holders;
   unsigned long long* slot_owner;
   int32_t* free_stack;
-  int32_t* ev_delta;
   uint32_t* stamp;
   DevState* st;
   uint64_t K;

@@ -660,106 +660,99 @@ constexpr int kEventLists = 8;
 struct EventBatch {
   const uint32_t* keys[kEventLists];
   const uint32_t* count[kEventLists];
-  int sign[kEventLists];
   int n;
 };
 
-// ev_delta[k] += sign of every listed key; the first batch of an advance
-// also clears the create / evict list counters.
-__global__ void events_add_kernel(EventBatch eb, int32_t* __restrict__ ev_delta, DevState* st,
-                                  int clear_counts) {
-  if (clear_counts && blockIdx.x == 0 && threadIdx.x == 0) {
-    st->n_create = 0;
-    st->n_evict = 0;
-  }
-  if (sort_failed(st)) return;
-  for (int l = 0; l < eb.n; ++l) {
-    const uint32_t n = *eb.count[l];
-    const uint32_t* keys = eb.keys[l];
-    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
-      atomicAdd(ev_delta + keys[i], eb.sign[l]);
-  }
+// The lists of a batch as one index space: pre[l] = keys before list l.
+__device__ __forceinline__ uint32_t batch_prefix(const EventBatch& eb, uint32_t (&pre)[kEventLists + 1]) {
+  pre[0] = 0;
+#pragma unroll
+  for (int l = 0; l < kEventLists; ++l) pre[l + 1] = pre[l] + (l < eb.n ? *eb.count[l] : 0u);
+  return pre[kEventLists];
 }
 
-// Net refcount change of every listed key (4 keys per thread per round),
-// appended to the create list (0 -> >0) or the evict list (>0 -> 0, if a
-// replica exists).  The order of a list is not specified.
-__global__ void events_apply_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* create_list,
-                                    uint32_t* evict_list) {
+// Key at flat index i (< total) of the batch.
+__device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32_t (&pre)[kEventLists + 1],
+                                              uint32_t i) {
+  int l = 0;
+#pragma unroll
+  for (int m = 1; m < kEventLists; ++m)
+    if (i >= pre[m]) l = m;
+  return eb.keys[l][i - pre[l]];
+}
+
+// Refcount transitions of one advance.  All lists whose window opens are
+// applied first (START, rc += 1; a key whose count was 0 is listed for
+// creation), then all lists whose window closes (rc -= 1; a key whose count
+// reaches 0 and that holds a replica is listed for eviction).  Every key of a
+// closing list had a positive count before the advance (its intent was
+// active), so with the openings first a key in both kinds of list never
+// crosses 0, and one atomic per listed key gives exactly the transitions of
+// the net change.  Four keys per thread and round; one list append per block
+// and round.  The order of a list is not specified.
+template <bool START>
+__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list) {
   if (sort_failed(s.st)) return;
   constexpr int Q = 4;
-  __shared__ uint32_t base_s[2];
-  uint16_t* rcw = s.rc + (uint64_t)w * s.K;
+  __shared__ uint32_t base_s;
+  uint32_t* rcw = s.rc + (uint64_t)w * s.K;
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
+  uint32_t* counter = START ? &s.st->n_create : &s.st->n_evict;
+  uint32_t pre[kEventLists + 1];
+  const uint32_t n = batch_prefix(eb, pre);
   const uint32_t stride = gridDim.x * blockDim.x * Q;
-  for (int l = 0; l < eb.n; ++l) {
-    const uint32_t n = *eb.count[l];
-    const uint32_t* keys = eb.keys[l];
-    for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
-      uint32_t k[Q];
-      int32_t d[Q], old[Q];
+  for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
+    uint32_t k[Q], old[Q];
+    bool hit[Q];
 #pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        const uint32_t i = b + q * blockDim.x + threadIdx.x;
-        k[q] = i < n ? keys[i] : 0u;
-      }
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      k[q] = i < n ? batch_key(eb, pre, i) : 0u;
+    }
 #pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        const uint32_t i = b + q * blockDim.x + threadIdx.x;
-        d[q] = i < n ? atomicExch(s.ev_delta + k[q], 0) : 0;
-      }
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      old[q] = 1u;   // neither transition
+      if (i < n) old[q] = START ? atomicAdd(rcw + k[q], 1u) : atomicSub(rcw + k[q], 1u);
+    }
 #pragma unroll
-      for (int q = 0; q < Q; ++q) old[q] = d[q] != 0 ? (int32_t)rcw[k[q]] : 0;
-      bool create[Q], evict[Q];
-#pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        create[q] = false;
-        evict[q] = false;
-        if (d[q] != 0) {
-          int32_t nw = old[q] + d[q];
-          if (nw < 0 || nw > 65535) {
-            set_error(s.st, ERR_REFCOUNT);
-            nw = nw < 0 ? 0 : 65535;
-          }
-          rcw[k[q]] = (uint16_t)nw;
-          create[q] = old[q] == 0 && nw > 0;
-          evict[q] = old[q] > 0 && nw == 0;
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      if (START) {
+        hit[q] = i < n && old[q] == 0u;
+        if (i < n && old[q] >= 65535u) set_error(s.st, ERR_REFCOUNT);
+      } else {
+        hit[q] = i < n && old[q] == 1u;
+        if (i < n && old[q] == 0u) {   // more closings than openings: undo, report
+          atomicAdd(rcw + k[q], 1u);
+          set_error(s.st, ERR_REFCOUNT);
         }
       }
-      // a key whose replica was never created (capacity exhausted) has nothing to destroy
+    }
+    // a key whose replica was never created (capacity exhausted) has nothing to destroy
+    if (!START) {
 #pragma unroll
       for (int q = 0; q < Q; ++q)
-        if (evict[q]) evict[q] = mapw[k[q]] >= 0;
-      // append: block-wide offsets, one atomic per list per block and round
-      uint32_t oc = 0, oe = 0;
-#pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        oc += create[q] ? 1u : 0u;
-        oe += evict[q] ? 1u : 0u;
-      }
-      uint32_t tc, te;
-      block_exclusive_scan2(oc, oe, tc, te);
-      if (threadIdx.x == 0) {
-        base_s[0] = tc ? atomicAdd(&s.st->n_create, tc) : 0u;
-        base_s[1] = te ? atomicAdd(&s.st->n_evict, te) : 0u;
-      }
-      __syncthreads();
-      oc += base_s[0];
-      oe += base_s[1];
-#pragma unroll
-      for (int q = 0; q < Q; ++q) {
-        if (create[q]) create_list[oc++] = k[q];
-        if (evict[q]) evict_list[oe++] = k[q];
-      }
-      __syncthreads();
+        if (hit[q]) hit[q] = mapw[k[q]] >= 0;
     }
+    uint32_t c = 0, unused = 0, total, t2;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) c += hit[q] ? 1u : 0u;
+    block_exclusive_scan2(c, unused, total, t2);
+    if (threadIdx.x == 0) base_s = total ? atomicAdd(counter, total) : 0u;
+    __syncthreads();
+    c += base_s;
+#pragma unroll
+    for (int q = 0; q < Q; ++q)
+      if (hit[q]) out_list[c++] = k[q];
+    __syncthreads();
   }
 }
 
 // evict: main[k] += acc[slot]; the freed slot goes on the stack at
-// free_top + i (every listed key holds a replica), so no atomics are needed.
-// R keys per row group at a time: list entries, slots, then the rows, each
-// as one round of independent loads.
+// free_top + i (every listed key holds a replica), so no list atomics are
+// needed.  R keys per row group at a time: list entries, slots, then the
+// pending rows, each as one round of independent loads.
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s, uint32_t w,
                                                                        const uint32_t* __restrict__ list) {
@@ -772,30 +765,44 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s
   float4* main4 = reinterpret_cast<float4*>(s.main);
   const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  for (uint64_t i0 = g * R; i0 < n; i0 += ng * R) {
-    uint32_t k[R];
-    int32_t sl[R];
+  const uint64_t step = ng * R;
+  // software-pipelined: a round loads the pending rows of its keys, the
+  // slots of the next round's keys and the list entries of the round after
+  auto load_keys = [&](uint64_t i0, uint32_t (&k)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) k[r] = i0 + r < n ? list[i0 + r] : 0u;
+  };
+  auto load_slots = [&](uint64_t i0, const uint32_t (&k)[R], int32_t (&sl)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? mapw[k[r]] : 0;
-    float4 m[R][C], ac[R][C];
+  };
+  uint32_t k[R], k1[R];
+  int32_t sl[R];
+  load_keys(g * R, k);
+  load_keys(g * R + step, k1);
+  load_slots(g * R, k, sl);
+  for (uint64_t i0 = g * R; i0 < n; i0 += step) {
+    float4 ac[R][C];
 #pragma unroll
     for (int r = 0; r < R; ++r)
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        const bool v = i0 + r < n && col < D4;
-        m[r][c] = v ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
-        ac[r][c] = v ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
+        ac[r][c] = (i0 + r < n && col < D4) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
       }
+    int32_t sl1[R];
+    uint32_t k2[R];
+    load_slots(i0 + step, k1, sl1);
+    load_keys(i0 + 2 * step, k2);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       if (i0 + r >= n) break;
+      // each listed key is evicted once, so main[k] has no other writer
+      // here: a vector atomic add gives main + acc without loading main
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        if (col < D4) main4[(uint64_t)k[r] * D4 + col] = f4add(m[r][c], ac[r][c]);
+        if (col < D4) atomicAdd(main4 + (uint64_t)k[r] * D4 + col, ac[r][c]);
       }
       if (lane == 0) {
         mapw[k[r]] = -1;
@@ -803,6 +810,12 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s
         s.slot_owner[sl[r]] = kEmptySlot;
         s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
       }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      k[r] = k1[r];
+      sl[r] = sl1[r];
+      k1[r] = k2[r];
     }
   }
 }
@@ -846,9 +859,10 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  for (uint64_t i0 = g * R; i0 < n; i0 += ng * R) {
-    uint32_t k[R];
-    int32_t sl[R];
+  const uint64_t step = ng * R;
+  // software-pipelined: a round loads the main rows of its keys and the list
+  // entries and slots of the next round together
+  auto load_entries = [&](uint64_t i0, uint32_t (&k)[R], int32_t (&sl)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       const bool v = i0 + r < n;
@@ -856,6 +870,11 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
       // slots popped from the top of the stack: lowest free slots come first
       sl[r] = v ? s.free_stack[base + (int32_t)(n - 1 - (i0 + r))] : 0;
     }
+  };
+  uint32_t k[R];
+  int32_t sl[R];
+  load_entries(g * R, k, sl);
+  for (uint64_t i0 = g * R; i0 < n; i0 += step) {
     float4 m[R][C];
 #pragma unroll
     for (int r = 0; r < R; ++r)
@@ -864,6 +883,9 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
         const uint32_t col = lane + c * G;
         m[r][c] = (i0 + r < n && col < D4) ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
       }
+    uint32_t k1[R];
+    int32_t sl1[R];
+    load_entries(i0 + step, k1, sl1);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       if (i0 + r >= n) break;
@@ -880,6 +902,11 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
         atomicOr(s.holders + k[r], 1u << w);
         s.slot_owner[sl[r]] = ((unsigned long long)w << 32) | k[r];
       }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      k[r] = k1[r];
+      sl[r] = sl1[r];
     }
   }
 }
@@ -1148,30 +1175,34 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
 
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
                    uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
-  // lists in batches of kEventLists: all refcount deltas first, then the
-  // transitions (a key in several lists changes once, by its net delta)
+  // all opening lists first, then all closing lists, in batches of kEventLists
   const uint64_t cap_blocks = (uint64_t)sms * 8;
   for (int pass = 0; pass < 2; ++pass) {
-    for (int i0 = 0; i0 < nlists; i0 += kEventLists) {
-      EventBatch eb{};
-      uint64_t cap = 0;
-      for (int l = 0; l < kEventLists && i0 + l < nlists; ++l) {
-        eb.keys[l] = lists[i0 + l].keys;
-        eb.count[l] = lists[i0 + l].count;
-        eb.sign[l] = lists[i0 + l].sign;
-        eb.n = l + 1;
-        if (lists[i0 + l].cap > cap) cap = lists[i0 + l].cap;
-      }
-      const uint64_t per = pass == 0 ? kThreads : 4 * kThreads;   // keys per block and round
-      uint64_t b = (cap + per - 1) / per;
+    const int sign = pass == 0 ? +1 : -1;
+    EventBatch eb{};
+    uint64_t cap = 0;
+    auto flush = [&]() {
+      if (eb.n == 0) return;
+      uint64_t b = (cap + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
       if (b > cap_blocks) b = cap_blocks;
       if (b == 0) b = 1;
       note_launches(1);
       if (pass == 0)
-        events_add_kernel<<<(unsigned)b, kThreads, 0, stream>>>(eb, s.ev_delta, s.st, i0 == 0 ? 1 : 0);
+        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list);
       else
-        events_apply_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list, evict_list);
+        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, evict_list);
+      eb = EventBatch{};
+      cap = 0;
+    };
+    for (int i = 0; i < nlists; ++i) {
+      if (lists[i].sign != sign) continue;
+      eb.keys[eb.n] = lists[i].keys;
+      eb.count[eb.n] = lists[i].count;
+      eb.n += 1;
+      cap += lists[i].cap;   // the kernel covers the batch's lists as one index space
+      if (eb.n == kEventLists) flush();
     }
+    flush();
   }
 }
 

@@ -200,6 +200,23 @@ def test_hot_key_spanning_many_chunks_and_determinism(gpu_lib):
     assert np.array_equal(outs[0], outs[1])
 
 
+def test_push_with_several_sort_subtiles_per_block(gpu_lib):
+    # 1.6M rows: more than one 2048-key sub-tile per block of the push's sort
+    # (at most 152 SMs x 4 blocks resident), and a hot key
+    K, D, W, n = 200_000, 4, 2, 1_600_000
+    rng = np.random.default_rng(11)
+    init = dyadic_init(K, D, 5)
+    keys = rng.integers(0, K, size=n)
+    keys[rng.random(n) < 0.05] = 777
+    d = (rng.integers(-64, 65, size=(n, D)) * 2.0 ** -12).astype(np.float32)
+    pm, ref = make_pair(gpu_lib, K, D, W, init)
+    for api in (pm, ref):
+        api.intent(0, np.arange(0, K, 3), 0, 2)
+        api.push(0, keys, d)
+    compare_full_state(pm, ref, K, W)
+    pm.close()
+
+
 def test_host_and_device_arguments_agree(gpu_lib):
     K, D, W = 3000, 32, 2
     init = dyadic_init(K, D, 9)
