@@ -91,33 +91,54 @@ mf_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ rows, const uin
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
   float4* d4 = reinterpret_cast<float4*>(o.drows);
   double lsum = 0.0;
-  for (uint64_t b = warp * GPW; b < n; b += nwarps * GPW) {
+  // software-pipelined: a round loads the rows of its cell, the slots of the
+  // next round's cell and the keys of the cell after
+  const uint64_t step = nwarps * GPW;
+  auto cell_keys = [&](uint64_t i, uint32_t& ku, uint32_t& kw) -> bool {   // both in range
+    ku = 0;
+    kw = 0;
+    if (i >= n) return false;
+    ku = rows[i];
+    kw = cols[i];
+    return ku < s.K && kw < s.K;
+  };
+  uint32_t ku0, kw0, ku1, kw1;
+  bool ok0 = cell_keys(warp * GPW + gi, ku0, kw0);
+  bool ok1 = cell_keys(warp * GPW + gi + step, ku1, kw1);
+  int32_t su0 = ok0 ? mapw[ku0] : -1, sw0 = ok0 ? mapw[kw0] : -1;
+  for (uint64_t b = warp * GPW; b < n; b += step) {
     const uint64_t i = b + gi;
     const bool in = i < n;
-    uint32_t ku = 0, kw = 0;
-    bool ok = false;
-    if (in) {
-      ku = rows[i];
-      kw = cols[i];
-      ok = ku < s.K && kw < s.K;
-      if (!ok && lane == 0) set_error(s.st, ERR_KEY_RANGE);
-    }
+    const uint32_t ku = ku0, kw = kw0;
+    const bool ok = ok0;
+    if (in && !ok && lane == 0) set_error(s.st, ERR_KEY_RANGE);
     float4 tu[C], tw[C], au[C], aw[C];
-    float part = 0.f;
-    if (ok) {
-      const float4* pu = row_ptr(s, mapw, ku);
-      const float4* pw = row_ptr(s, mapw, kw);
+    {
+      const float4* pu = su0 >= 0 ? reinterpret_cast<const float4*>(s.val) + (uint64_t)su0 * D4
+                                  : reinterpret_cast<const float4*>(s.main) + (uint64_t)ku * D4;
+      const float4* pw = sw0 >= 0 ? reinterpret_cast<const float4*>(s.val) + (uint64_t)sw0 * D4
+                                  : reinterpret_cast<const float4*>(s.main) + (uint64_t)kw * D4;
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        const bool cv = col < dim4;
+        const bool cv = ok && col < dim4;
         tu[c] = cv ? pu[col] : f4zero();
         tw[c] = cv ? pw[col] : f4zero();
         au[c] = (cv && adagrad) ? pu[dim4 + col] : f4zero();
         aw[c] = (cv && adagrad) ? pw[dim4 + col] : f4zero();
-        part += dot4(tu[c], tw[c]);
       }
     }
+    // the next cell's slots and the keys of the cell after, issued before
+    // this cell's rows are used
+    su0 = ok1 ? mapw[ku1] : -1;
+    sw0 = ok1 ? mapw[kw1] : -1;
+    ku0 = ku1;
+    kw0 = kw1;
+    ok0 = ok1;
+    ok1 = cell_keys(i + 2 * step, ku1, kw1);
+    float part = 0.f;
+#pragma unroll
+    for (int c = 0; c < C; ++c) part += dot4(tu[c], tw[c]);
     const float dot = group_sum<G>(part);
     if (!in) continue;
     if (!ok) {
@@ -198,27 +219,41 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
       Tre[c] = f4zero();
       Tim[c] = f4zero();
     }
-    // tails: j = 0 is the true tail (label +1), j >= 1 the negatives (label -1)
-    for (uint32_t j0 = 0; j0 < 1 + n_neg; j0 += U) {
-      uint32_t kx[U];
-      bool vx[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const uint32_t j = j0 + u;
-        kx[u] = j == 0 ? kt : (j <= n_neg ? negs[i * n_neg + (j - 1)] : kNoKey);
-        vx[u] = j <= n_neg && kx[u] < s.K;
-        if (j <= n_neg && kx[u] >= s.K && lane == 0) set_error(s.st, ERR_KEY_RANGE);
+    // tails: j = 0 is the true tail (label +1), j >= 1 the negatives (label
+    // -1); software-pipelined: a round loads the tail rows of U indices, the
+    // slots of the next U and the keys of the U after
+    const uint32_t J = 1 + n_neg;
+    auto tail_key = [&](uint32_t j) -> uint32_t {   // kNoKey: skipped
+      if (j >= J) return kNoKey;
+      const uint32_t k = j == 0 ? kt : negs[i * n_neg + (j - 1)];
+      if (k >= s.K) {
+        if (lane == 0) set_error(s.st, ERR_KEY_RANGE);
+        return kNoKey;
       }
+      return k;
+    };
+    uint32_t k0[U], k1[U];
+    int32_t s0[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      k0[u] = tail_key(u);
+      k1[u] = tail_key(U + u);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) s0[u] = k0[u] != kNoKey ? mapw[k0[u]] : -1;
+    for (uint32_t j0 = 0; j0 < J; j0 += U) {
       float4 tre[U][CC], tim[U][CC], are[U][CC], aim[U][CC];
       float part[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const float4* pt = vx[u] ? row_ptr(s, mapw, kx[u]) : nullptr;
+        const bool vx = k0[u] != kNoKey;
+        const float4* pt = s0[u] >= 0 ? reinterpret_cast<const float4*>(s.val) + (uint64_t)s0[u] * D4
+                                      : reinterpret_cast<const float4*>(s.main) + (uint64_t)k0[u] * D4;
         part[u] = 0.f;
 #pragma unroll
         for (int c = 0; c < CC; ++c) {
           const uint32_t q = lane + 32 * c;
-          const bool cv = vx[u] && q < h4;
+          const bool cv = vx && q < h4;
           tre[u][c] = cv ? pt[q] : f4zero();
           tim[u][c] = cv ? pt[h4 + q] : f4zero();
           are[u][c] = cv ? pt[2 * h4 + q] : f4zero();
@@ -226,13 +261,19 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
           part[u] += dot4(xre[c], tre[u][c]) + dot4(xim[c], tim[u][c]);
         }
       }
+      int32_t s1[U];
+      uint32_t k2[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) s1[u] = k1[u] != kNoKey ? mapw[k1[u]] : -1;
+#pragma unroll
+      for (int u = 0; u < U; ++u) k2[u] = tail_key(j0 + 2 * U + u);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const uint32_t j = j0 + u;
         const float phi = group_sum<32>(part[u]);
-        if (j > n_neg) continue;
+        if (j >= J) continue;
         const uint64_t row = base + (j == 0 ? 2 : 2 + j);
-        if (!vx[u]) {
+        if (k0[u] == kNoKey) {
           if (lane == 0) o.dkeys[row] = kNoKey;
           continue;
         }
@@ -251,7 +292,13 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
             d4[row * D4 + 3 * h4 + q] = sq4(gim);
           }
         }
-        if (lane == 0) o.dkeys[row] = kx[u];
+        if (lane == 0) o.dkeys[row] = k0[u];
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        k0[u] = k1[u];
+        s0[u] = s1[u];
+        k1[u] = k2[u];
       }
     }
     // head and relation: gradients are linear in T = sum_j coef_j t_j
@@ -319,60 +366,91 @@ sgns_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ centres, cons
       v[c] = col < D4 ? pv[col] : f4zero();
       gv[c] = f4zero();
     }
-    for (uint32_t j = 0; j < n_ctx; ++j) {
+    // the centre's rows in one index space t = j * (1 + n_neg) + q (q = 0:
+    // the context word, q >= 1: its negatives), software-pipelined: a round
+    // loads the rows of U indices, the slots of the next U and the tokens of
+    // the U after, so one memory latency per round
+    const uint32_t per_ctx = 1 + n_neg;
+    const uint32_t T = n_ctx * per_ctx;
+    auto token = [&](uint32_t t) -> uint32_t {   // the row's key, kNoKey when it is skipped
+      if (t >= T) return kNoKey;
+      const uint32_t j = t / per_ctx, q = t - j * per_ctx;
       const uint32_t oc = contexts[i * n_ctx + j];
-      const uint64_t rb = base + 1 + (uint64_t)j * (1 + n_neg);
-      if (oc == kNoKey || oc >= vocab) {
-        if (oc != kNoKey && lane == 0) set_error(s.st, ERR_KEY_RANGE);
-        for (uint64_t q = lane; q < 1 + (uint64_t)n_neg; q += 32) o.dkeys[rb + q] = kNoKey;
-        continue;
+      if (oc == kNoKey) return kNoKey;
+      if (oc >= vocab) {
+        if (q == 0 && lane == 0) set_error(s.st, ERR_KEY_RANGE);
+        return kNoKey;
       }
-      for (uint32_t q0 = 0; q0 < 1 + n_neg; q0 += U) {
-        uint32_t kx[U];
-        bool vx[U];
+      const uint32_t tok = q == 0 ? oc : negs[(i * n_ctx + j) * n_neg + (q - 1)];
+      if (tok >= vocab) {
+        if (lane == 0) set_error(s.st, ERR_KEY_RANGE);
+        return kNoKey;
+      }
+      return vocab + tok;
+    };
+    uint32_t k0[U], k1[U];
+    int32_t s0[U];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const uint32_t q = q0 + u;
-          uint32_t tok = kNoKey;
-          if (q == 0) tok = oc;
-          else if (q <= n_neg) tok = negs[(i * n_ctx + j) * n_neg + (q - 1)];
-          vx[u] = q <= n_neg && tok < vocab;
-          if (q <= n_neg && tok >= vocab && lane == 0) set_error(s.st, ERR_KEY_RANGE);
-          kx[u] = vx[u] ? vocab + tok : kNoKey;
+    for (int u = 0; u < U; ++u) {
+      k0[u] = token(u);
+      k1[u] = token(U + u);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) s0[u] = k0[u] != kNoKey ? mapw[k0[u]] : -1;
+    for (uint32_t t0 = 0; t0 < T; t0 += U) {
+      float4 x[U][C];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const bool vx = k0[u] != kNoKey;
+        const float4* px = s0[u] >= 0 ? reinterpret_cast<const float4*>(s.val) + (uint64_t)s0[u] * D4
+                                      : reinterpret_cast<const float4*>(s.main) + (uint64_t)k0[u] * D4;
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + 32 * c;
+          x[u][c] = (vx && col < D4) ? px[col] : f4zero();
         }
-        float4 x[U][C];
-        float part[U];
+      }
+      // the next round's slots and the tokens of the round after, issued
+      // before this round's rows are used
+      int32_t s1[U];
+      uint32_t k2[U];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const float4* px = vx[u] ? row_ptr(s, mapw, kx[u]) : nullptr;
-          part[u] = 0.f;
+      for (int u = 0; u < U; ++u) s1[u] = k1[u] != kNoKey ? mapw[k1[u]] : -1;
 #pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + 32 * c;
-            x[u][c] = (vx[u] && col < D4) ? px[col] : f4zero();
-            part[u] += dot4(x[u][c], v[c]);
-          }
+      for (int u = 0; u < U; ++u) k2[u] = token(t0 + 2 * U + u);
+      float part[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        part[u] = 0.f;
+#pragma unroll
+        for (int c = 0; c < C; ++c) part[u] += dot4(x[u][c], v[c]);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const uint32_t t = t0 + u;
+        const float sc = group_sum<32>(part[u]);
+        if (t >= T) continue;
+        const uint64_t row = base + 1 + t;
+        if (k0[u] == kNoKey) {
+          if (lane == 0) o.dkeys[row] = kNoKey;
+          continue;
         }
+        const bool positive = t % per_ctx == 0;
+        const float coef = positive ? -sigmoid_f(-sc) : sigmoid_f(sc);
+        if (lane == 0) lsum += (double)(positive ? softplus_f(-sc) : softplus_f(sc));
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const uint32_t q = q0 + u;
-          const float sc = group_sum<32>(part[u]);
-          if (q > n_neg) continue;
-          const uint64_t row = rb + q;
-          if (!vx[u]) {
-            if (lane == 0) o.dkeys[row] = kNoKey;
-            continue;
-          }
-          const float coef = q == 0 ? -sigmoid_f(-sc) : sigmoid_f(sc);
-          if (lane == 0) lsum += (double)(q == 0 ? softplus_f(-sc) : softplus_f(sc));
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + 32 * c;
-            gv[c] = f4fma(x[u][c], coef, gv[c]);
-            if (col < D4) d4[row * D4 + col] = f4scale(v[c], -lr * coef);
-          }
-          if (lane == 0) o.dkeys[row] = kx[u];
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + 32 * c;
+          gv[c] = f4fma(x[u][c], coef, gv[c]);
+          if (col < D4) d4[row * D4 + col] = f4scale(v[c], -lr * coef);
         }
+        if (lane == 0) o.dkeys[row] = k0[u];
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        k0[u] = k1[u];
+        s0[u] = s1[u];
+        k1[u] = k2[u];
       }
     }
 #pragma unroll
