@@ -231,6 +231,14 @@ adapm_status adapm_kernel_launches(uint64_t* out);
 /* Message for the last error returned on this context ("" if none). */
 const char* adapm_last_error(adapm_ctx* ctx);
 
+/* Fault injection for tests of the bounded device waits (no GPU fault is
+ * involved): the next push of this context sorts its keys in a launch whose
+ * first grid barrier waits for arrivals that never come.  That wait gives up
+ * after about a second, the push leaves the store untouched, and
+ * adapm_wait returns ADAPM_ETIMEOUT; the context is unusable afterwards,
+ * other contexts are unaffected. */
+adapm_status adapm_debug_fail_next_barrier(adapm_ctx* ctx);
+
 #ifdef __cplusplus
 }
 #endif

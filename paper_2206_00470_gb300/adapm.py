@@ -27,6 +27,7 @@ EXPORTS = [
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
     "adapm_refcounts", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
     "adapm_profile_read", "adapm_kernel_launches", "adapm_push_noalloc", "adapm_last_error",
+    "adapm_debug_fail_next_barrier",
 ]
 
 
@@ -97,6 +98,7 @@ def load(path=LIB_PATH):
         "adapm_profile_read": [P, P, P],
         "adapm_kernel_launches": [ctypes.POINTER(U64)],
         "adapm_push_noalloc": [P, U32, P, U64, P],
+        "adapm_debug_fail_next_barrier": [P],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -245,6 +247,10 @@ class ParameterManager:
         if d.n != k.n * self.D:
             raise ValueError("deltas must hold len(keys) * value_len floats")
         self._check(self._lib.adapm_push_noalloc(self._h, worker, k.ptr, k.n, d.ptr))
+
+    def debug_fail_next_barrier(self):
+        """Test hook: the next push's sort gives up its grid-barrier wait (ADAPM_ETIMEOUT at wait)."""
+        self._check(self._lib.adapm_debug_fail_next_barrier(self._h))
 
     def sync(self):
         self._check(self._lib.adapm_sync(self._h))

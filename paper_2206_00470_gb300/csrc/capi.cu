@@ -517,6 +517,13 @@ adapm_status adapm_sync(adapm_ctx* ctx) {
   return check_launch(ctx, "sync");
 }
 
+adapm_status adapm_debug_fail_next_barrier(adapm_ctx* ctx) {
+  if (!ctx) return ADAPM_EINVAL;
+  // the next sort expects arrivals far beyond those that can happen
+  ctx->bar_base += 1ull << 40;
+  return ADAPM_OK;
+}
+
 adapm_status adapm_wait(adapm_ctx* ctx) {
   if (!ctx) return ADAPM_EINVAL;
   if (ctx->broken) return fail(ctx, ADAPM_ECUDA, "context unusable after an earlier CUDA error");

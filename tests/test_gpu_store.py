@@ -8,7 +8,7 @@ oracle with the same seeded call sequence and compares:
   * with gaussian deltas: |gpu - oracle| <= 1e-5 * M + 1e-30 per element,
     M = the same quantity computed on |init| and |deltas| (the sum of the
     magnitudes of every contribution to that element).
-Sizes span several 2048-key sort tiles, many push chunks and ragged tails.
+Sizes span several sort sub-tiles, many push chunks and ragged tails.
 """
 import numpy as np
 import pytest
@@ -92,7 +92,7 @@ CASES = [
     # K, D, W, max_batch, n_ops
     (40, 4, 3, 12, 160),
     (300, 16, 4, 700, 60),
-    (5000, 64, 3, 6000, 40),      # several sort tiles, ragged tails, many push chunks
+    (5000, 64, 3, 6000, 40),      # several sort sub-tiles, ragged tails, many push chunks
     (900, 200, 2, 2500, 30),
     (700, 300, 2, 1500, 25),
     (500, 512, 2, 1200, 25),
@@ -200,10 +200,12 @@ def test_hot_key_spanning_many_chunks_and_determinism(gpu_lib):
     assert np.array_equal(outs[0], outs[1])
 
 
-def test_push_with_several_sort_subtiles_per_block(gpu_lib):
-    # 1.6M rows: more than one 2048-key sub-tile per block of the push's sort
-    # (at most 152 SMs x 4 blocks resident), and a hot key
-    K, D, W, n = 200_000, 4, 2, 1_600_000
+@pytest.mark.parametrize("n", [200_000, 400_000, 1_600_000])
+def test_push_sizes_across_the_sort_layouts(gpu_lib, n):
+    # the push's sort at 200k rows: 1024-key sub-tiles, digit rows scanned by
+    # four warps; 400k: 2048-key sub-tiles, four warps; 1.6M: more than one
+    # sub-tile per block (at most 152 SMs x 4 blocks resident); a hot key
+    K, D, W = 200_000, 4, 2
     rng = np.random.default_rng(11)
     init = dyadic_init(K, D, 5)
     keys = rng.integers(0, K, size=n)
