@@ -4,8 +4,10 @@
 // owning columns lane, lane+G, ..., lane+(C-1)G of a row (D4 = D/4 <= G*C).
 // Kernels are persistent grids (a multiple of the SM count) with several
 // independent rows in flight per group (R-way unrolled address chains:
-// key -> slot -> row), which is what an HBM-bound gather needs.
+// key -> slot -> row, software-pipelined where registers allow), which is
+// what an HBM-bound gather needs.
 //
+//   intent      the distinct keys of one call (hash set + stamps)       (Sec. 3)
 //   pull        out[i] = replica of keys[i] at worker w, else main       (Sec. 5.1)
 //   push        sorted (key, position) pairs are split into fixed chunks;
 //               each group sums the delta rows of every key segment of its
@@ -13,8 +15,9 @@
 //               replica (value and pending updates) or to main (Sec. 4,
 //               App. B.1.2); segments cut by a chunk boundary leave partial
 //               sums that one owner combines in chunk order (fix-up)
-//   events      net refcount change per key of one advance, transitions
-//               0 -> >0 (create) and >0 -> 0 (evict)                    (Sec. 3)
+//   events      refcount +1 for every key of the opening intent lists,
+//               then -1 for the closing ones; transitions 0 -> 1 (create)
+//               and 1 -> 0 (evict)                                      (Sec. 3)
 //   evict       main += pending updates; free the slot                 (Sec. 4.1)
 //   create      val = main, pending = 0; take a slot                   (Sec. 4.1)
 //   sync        main += sum of all holders' pending updates (ascending
@@ -653,7 +656,7 @@ __global__ void __launch_bounds__(kThreads) intent_dedup_kernel(Store s, const u
 }
 
 // ---------------------------------------------------------------------------
-// intent events -> refcounts -> create / evict lists
+// advance: intent lists -> refcounts -> create / evict lists
 // ---------------------------------------------------------------------------
 // Up to kEventLists intent lists handled by one launch.
 constexpr int kEventLists = 8;
