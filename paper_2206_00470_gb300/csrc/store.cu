@@ -435,12 +435,13 @@ __global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs 
 }
 
 // Hot keys: a segment whose pieces run over more than kShortSpan further
-// spans.  Its head pieces j+1 .. m_end are cut into work items of kLongSub
+// chunks.  Its head pieces j+1 .. m_end are cut into work items of kLongSub
 // pieces, spread over all blocks; a block sums its item (groups take strided
 // pieces in increasing order, then the group sums in group order) into
-// long_parts.  The block that finishes an entry's last item adds the tail
-// piece and the item sums in item order and applies the total.  Every sum has
-// a fixed order, so the result does not depend on which block finishes last.
+// long_parts.  The block that finishes an entry's last item sums the item
+// sums the same way (groups take strided items, then group order), adds the
+// tail piece and applies the total.  Every sum has a fixed order, so the
+// result does not depend on which block finishes last.
 constexpr uint32_t kLongSub = 32;
 constexpr uint32_t kLongSmem = 1024;   // long-list entries whose item bases sit in shared memory
 
@@ -557,33 +558,43 @@ __global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a
     __syncthreads();
     if (threadIdx.x == 0) s_last = atomicAdd(long_list + 4 * e + 2, 1u) == (uint32_t)(ns - 1);
     __syncthreads();
-    if (s_last && gi == 0) {
+    if (s_last) {   // block-uniform
+      // the entry's item sums: group g adds items g, g + NG, ... in order,
+      // then group 0 adds the tail piece and the group sums in group order
       __threadfence();
-      const uint32_t kl = a.skeys[(j + 1) * CH - 1];
-      float4 tot[C];
+      float4 acc2[C];
 #pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
-      }
-      // the item sums in item order, several loads in flight
-      constexpr int UB = 8 / C > 0 ? 8 / C : 1;
-      for (uint64_t i0 = 0; i0 < ns; i0 += UB) {
+      for (int c = 0; c < C; ++c) acc2[c] = f4zero();
+      constexpr int UB = 4 / C > 0 ? 4 / C : 1;
+      for (uint64_t i0 = gi; i0 < ns; i0 += (uint64_t)NG * UB) {
         float4 t[UB][C];
 #pragma unroll
         for (int u = 0; u < UB; ++u)
 #pragma unroll
           for (int c = 0; c < C; ++c) {
             const uint32_t col = lane + c * G;
-            t[u][c] = (i0 + u < ns && col < D4) ? __ldcg(lp4 + (base + i0 + u) * D4 + col) : f4zero();
+            const uint64_t it2 = i0 + (uint64_t)u * NG;
+            t[u][c] = (it2 < ns && col < D4) ? __ldcg(lp4 + (base + it2) * D4 + col) : f4zero();
           }
 #pragma unroll
         for (int u = 0; u < UB; ++u)
-          if (i0 + u < ns)
 #pragma unroll
-            for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+          for (int c = 0; c < C; ++c) acc2[c] = f4add(acc2[c], t[u][c]);
       }
-      apply_sum<C>(s, mapw, kl, tot, lane, G);
+#pragma unroll
+      for (int c = 0; c < C; ++c) part[gi][lane + c * G] = acc2[c];
+      __syncthreads();
+      if (gi == 0) {
+        const uint32_t kl = a.skeys[(j + 1) * CH - 1];
+        float4 tot[C];
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
+          for (int g2 = 0; g2 < NG; ++g2) tot[c] = f4add(tot[c], part[g2][lane + c * G]);
+        }
+        apply_sum<C>(s, mapw, kl, tot, lane, G);
+      }
     }
     __syncthreads();
   }
