@@ -3,8 +3,9 @@
 TEST INFRASTRUCTURE ONLY (see oracle/__init__.py).
 
 State follows the paper's description of AdaPM with worker slots in the role
-of nodes and replication always chosen (the paper's "AdaPM w/o relocation"
-variant, Sec. 5.5):
+of nodes.  By default replication is always chosen (the paper's "AdaPM w/o
+relocation" variant, Sec. 5.5); with relocation=True the full decision rule
+of Sec. 4.1 applies (see "Relocation" below):
 
   main[K][D]        the main copy of every parameter (fp32)
   clock[w]          worker w's logical clock C^w, starts at 0 (Sec. 3)
@@ -36,6 +37,27 @@ Definitions
     acc = 0 (App. B.1.2: the owner merges the updates and propagates them to
     the replica holders; sending only unseen versions gives the same values).
 
+Relocation (Sec. 4.1 and App. B.3, "relocate only when exactly one node has
+active intent"; scenarios of Fig. 4b-d and Fig. 10a)
+  * Every key has an owner: a worker slot, or its home (-1) before any
+    worker has held it.  The owner accesses the main copy directly and holds
+    no replica; every other worker with active intent holds a replica.
+  * Whenever exactly one worker has active intent for a key and it is not the
+    owner, the key is relocated to it: if that worker holds a replica, the
+    replica is destroyed first (its pending updates merged into main, as on
+    any destruction), then the worker becomes the owner.  Ownership stays
+    where it is when the owner's intent expires, while several workers have
+    active intent, and while nobody has.
+  * Within one call only the calling worker's active set changes, so a key
+    is either joined or left by that worker.  Left keys (ascending) go first:
+    the worker's replica is destroyed, then a sole remaining active worker
+    becomes the owner.  Joined keys (ascending) follow: with no other active
+    worker the caller becomes the owner, otherwise it gets a replica unless
+    it is the owner already.
+  * pull, push and sync are unchanged: the owner holds no replica, so its
+    reads and writes go to main; a sole active worker therefore sees other
+    workers' writes at once.
+
 Arithmetic: every sum runs in fp64 and is rounded to fp32 once when stored.
 """
 import numpy as np
@@ -50,17 +72,21 @@ def _f32(x):
 
 
 class ParameterManagerOracle:
-    def __init__(self, num_keys, value_len, num_workers, init):
+    def __init__(self, num_keys, value_len, num_workers, init, relocation=False):
         init = np.asarray(init, dtype=np.float32)
         if init.shape != (num_keys, value_len):
             raise OracleError("init must have shape (num_keys, value_len)")
         self.K = int(num_keys)
         self.D = int(value_len)
         self.W = int(num_workers)
+        self.relocation = bool(relocation)
         self.main = init.copy()
         self.clock = [0] * self.W
         self.intents = [[] for _ in range(self.W)]   # entries: (frozenset keys, start, end)
         self.replicas = [dict() for _ in range(self.W)]
+        self.active = [set() for _ in range(self.W)]  # A_w(C^w) as of w's last call
+        self.owner = np.full(self.K, -1, dtype=np.int64)
+        self.created = self.destroyed = self.relocations = 0
 
     # -- argument checks ---------------------------------------------------
     def _check_worker(self, w):
@@ -90,15 +116,51 @@ class ParameterManagerOracle:
         c = self.clock[w]
         return sum(1 for keys, s, e in self.intents[w] if self._is_active(s, e, c) and k in keys)
 
+    def _create(self, w, k):
+        self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+        self.created += 1
+
+    def _destroy(self, w, k):
+        val, acc = self.replicas[w].pop(k)
+        self.main[k] = _f32(self.main[k].astype(np.float64) + acc.astype(np.float64))
+        self.destroyed += 1
+
+    def _relocate(self, k, w):
+        """Make w the owner of k; a replica it holds is merged into main first."""
+        if self.owner[k] == w:
+            return
+        if k in self.replicas[w]:
+            self._destroy(w, k)
+        self.owner[k] = w
+        self.relocations += 1
+
+    def _others_active(self, w, k):
+        return [v for v in range(self.W) if v != w and k in self.active[v]]
+
     def _reconcile(self, w):
-        """Make R_w equal A_w(C^w): destroy, then create, each in ascending key order."""
-        active = self.active_set(w)
-        held = set(self.replicas[w])
-        for k in sorted(held - active):
-            val, acc = self.replicas[w].pop(k)
-            self.main[k] = _f32(self.main[k].astype(np.float64) + acc.astype(np.float64))
-        for k in sorted(active - held):
-            self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+        now = self.active_set(w)
+        if self.relocation:
+            before = self.active[w]
+            for k in sorted(before - now):            # w's intent for k expired
+                if k in self.replicas[w]:
+                    self._destroy(w, k)
+                others = self._others_active(w, k)
+                if len(others) == 1:
+                    self._relocate(k, others[0])
+            for k in sorted(now - before):            # w's intent for k became active
+                others = self._others_active(w, k)
+                if not others:
+                    self._relocate(k, w)
+                elif self.owner[k] != w:
+                    self._create(w, k)
+        else:
+            # R_w := A_w(C^w): destroy, then create, each in ascending key order
+            held = set(self.replicas[w])
+            for k in sorted(held - now):
+                self._destroy(w, k)
+            for k in sorted(now - held):
+                self._create(w, k)
+        self.active[w] = now
         # expired intents can never become active again (clocks only rise)
         c = self.clock[w]
         self.intents[w] = [(keys, s, e) for keys, s, e in self.intents[w] if e > c]
@@ -177,3 +239,8 @@ class ParameterManagerOracle:
     def read_main(self, keys):
         keys = self._check_keys(keys)
         return self.main[keys].copy()
+
+    def owners(self, keys):
+        """Owner worker of each key, -1 for a key still at its home."""
+        keys = self._check_keys(keys)
+        return self.owner[keys].copy()
