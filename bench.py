@@ -45,25 +45,27 @@ METRIC = "pulled+pushed keys/s and training samples/s on 1 GB300; % of HBM roofl
 # DRAM bytes (read + write) of the push scatter kernels (push_chunks + push_fixup + push_long) per
 # pushed row, per workload, from the full ncu captures summarised in profiles/ (each on a smaller case
 # of the same workload, scaled by rows); a figure stands for the kernels only while their source is the
-# one captured (source_digest: first 16 hex digits of the sha256 of its code without comments), otherwise
+# one captured (source_digest: first 16 hex digits of the sha256 of their code without comments), otherwise
 # the traffic is reported as null.
-PUSH_SOURCE = "paper_2206_00470_gb300/csrc/store.cu"
+PUSH_SOURCES = ("paper_2206_00470_gb300/csrc/push.cu", "paper_2206_00470_gb300/csrc/rowgroup.cuh")
 PUSH_TRAFFIC = {
-    "mf": {"bytes_per_row": 79.02e6 / 65536, "sha256_16": "dd9908467d255e88"},   # profiles/push_scatter_mf_2Mx200K.md
+    "mf": {"bytes_per_row": 79.213e6 / 65536, "sha256_16": "f902f353c30b86b9"},   # profiles/push_scatter_mf_2Mx200K.md
     "micro": {"bytes_per_row": None, "sha256_16": None},
 }
 
 
-def source_digest(path):
-    """sha256 (16 hex digits) of a CUDA source with its // comments and blank lines removed, so that
+def source_digest(paths):
+    """sha256 (16 hex digits) of CUDA sources with their // comments and blank lines removed, so that
     a change to comments alone does not retire a recorded capture."""
     import hashlib
     import re
-    with open(path) as f:
-        text = f.read()
-    lines = [re.sub(r"//.*$", "", ln).rstrip() for ln in text.splitlines()]
-    code = "\n".join(ln for ln in lines if ln.strip())
-    return hashlib.sha256(code.encode()).hexdigest()[:16]
+    code = []
+    for path in paths:
+        with open(path) as f:
+            text = f.read()
+        lines = [re.sub(r"//.*$", "", ln).rstrip() for ln in text.splitlines()]
+        code.append("\n".join(ln for ln in lines if ln.strip()))
+    return hashlib.sha256("\n".join(code).encode()).hexdigest()[:16]
 
 
 def recorded_traffic(workload, rows_per_launch):
@@ -71,7 +73,7 @@ def recorded_traffic(workload, rows_per_launch):
     if not rec or rec["bytes_per_row"] is None:
         return None
     try:
-        digest = source_digest(os.path.join(ROOT, PUSH_SOURCE))
+        digest = source_digest([os.path.join(ROOT, p) for p in PUSH_SOURCES])
     except OSError:
         return None
     if digest != rec["sha256_16"]:

@@ -1,0 +1,402 @@
+// Intent bookkeeping on the device: the distinct keys of an Intent call, and
+// the refcount events of advanceClock with the replicas they create and
+// destroy (Sec. 3, Sec. 4.1).
+//
+//   intent      the distinct keys of one call (hash set + stamps)       (Sec. 3)
+//   events      refcount +1 for every key of the opening intent lists,
+//               then -1 for the closing ones; transitions 0 -> 1 (create)
+//               and 1 -> 0 (evict)                                      (Sec. 3)
+//   evict       main += pending updates; free the slot                 (Sec. 4.1)
+//   create      val = main, pending = 0; take a slot                   (Sec. 4.1)
+#include "internal.cuh"
+#include "rowgroup.cuh"
+#include "store_launch.cuh"
+
+namespace adapm {
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// intent: the distinct keys of one call (Sec. 3: an intent names a set of
+// parameters, so a key listed twice in one call counts once)
+// ---------------------------------------------------------------------------
+constexpr int kDedupItems = 8;
+constexpr int kDedupTile = kThreads * kDedupItems;   // keys per block and round
+constexpr int kDedupTab = 2 * kDedupTile;            // shared hash table, half full at most
+
+// Each block takes tiles of 2048 keys: a shared-memory hash set (open
+// addressing) keeps the first copy of every key of the tile, and an exchange
+// on the key's stamp keeps the first copy over all tiles (stamp == tag once
+// some copy has been listed).  One atomic per block and round appends.
+__global__ void __launch_bounds__(kThreads) intent_dedup_kernel(Store s, const uint32_t* __restrict__ keys,
+                                                                uint64_t n, uint32_t tag,
+                                                                uint32_t* __restrict__ out, uint32_t* count) {
+  __shared__ uint32_t tab[kDedupTab];
+  __shared__ uint32_t base_s;
+  bool bad = false;
+  for (uint64_t t0 = (uint64_t)blockIdx.x * kDedupTile; t0 < n;
+       t0 += (uint64_t)gridDim.x * kDedupTile) {   // block-uniform trip count
+    for (int i = threadIdx.x; i < kDedupTab; i += kThreads) tab[i] = kNoKey;
+    __syncthreads();
+    uint32_t k[kDedupItems];
+    bool first[kDedupItems];
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) {
+      const uint64_t i = t0 + (uint64_t)it * kThreads + threadIdx.x;
+      k[it] = i < n ? __ldg(keys + i) : kNoKey;
+      if (i < n && k[it] >= s.K) {
+        bad = true;
+        k[it] = kNoKey;
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) {
+      first[it] = false;
+      if (k[it] == kNoKey) continue;
+      uint32_t h = (k[it] * 0x9E3779B1u) >> (32 - 12);   // 12 bits: kDedupTab = 4096
+      for (int probe = 0; probe < kDedupTab; ++probe) {
+        const uint32_t old = atomicCAS(&tab[h], kNoKey, k[it]);
+        if (old == kNoKey) {
+          first[it] = true;
+          break;
+        }
+        if (old == k[it]) break;
+        h = (h + 1) & (kDedupTab - 1);
+      }
+    }
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it)
+      if (first[it]) first[it] = atomicExch(s.stamp + k[it], tag) != tag;
+    uint32_t c = 0, unused = 0, total, t2;
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it) c += first[it] ? 1u : 0u;
+    block_exclusive_scan2(c, unused, total, t2);
+    if (threadIdx.x == 0) base_s = total ? atomicAdd(count, total) : 0u;
+    __syncthreads();
+    c += base_s;
+#pragma unroll
+    for (int it = 0; it < kDedupItems; ++it)
+      if (first[it]) out[c++] = k[it];
+    __syncthreads();
+  }
+  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(s.st, ERR_KEY_RANGE);
+}
+
+// ---------------------------------------------------------------------------
+// advance: intent lists -> refcounts -> create / evict lists
+// ---------------------------------------------------------------------------
+// Up to kEventLists intent lists handled by one launch.
+constexpr int kEventLists = 8;
+struct EventBatch {
+  const uint32_t* keys[kEventLists];
+  const uint32_t* count[kEventLists];
+  int n;
+};
+
+// The lists of a batch as one index space: pre[l] = keys before list l.
+__device__ __forceinline__ uint32_t batch_prefix(const EventBatch& eb, uint32_t (&pre)[kEventLists + 1]) {
+  pre[0] = 0;
+#pragma unroll
+  for (int l = 0; l < kEventLists; ++l) pre[l + 1] = pre[l] + (l < eb.n ? *eb.count[l] : 0u);
+  return pre[kEventLists];
+}
+
+// Key at flat index i (< total) of the batch.
+__device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32_t (&pre)[kEventLists + 1],
+                                              uint32_t i) {
+  int l = 0;
+#pragma unroll
+  for (int m = 1; m < kEventLists; ++m)
+    if (i >= pre[m]) l = m;
+  return eb.keys[l][i - pre[l]];
+}
+
+// Refcount transitions of one advance.  All lists whose window opens are
+// applied first (START, rc += 1; a key whose count was 0 is listed for
+// creation), then all lists whose window closes (rc -= 1; a key whose count
+// reaches 0 and that holds a replica is listed for eviction).  Every key of a
+// closing list had a positive count before the advance (its intent was
+// active), so with the openings first a key in both kinds of list never
+// crosses 0, and one atomic per listed key gives exactly the transitions of
+// the net change.  Four keys per thread and round; one list append per block
+// and round.  The order of a list is not specified.
+template <bool START>
+__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list) {
+  if (sort_failed(s.st)) return;
+  constexpr int Q = 4;
+  __shared__ uint32_t base_s;
+  uint32_t* rcw = s.rc + (uint64_t)w * s.K;
+  const int32_t* mapw = s.map + (uint64_t)w * s.K;
+  uint32_t* counter = START ? &s.st->n_create : &s.st->n_evict;
+  uint32_t pre[kEventLists + 1];
+  const uint32_t n = batch_prefix(eb, pre);
+  const uint32_t stride = gridDim.x * blockDim.x * Q;
+  for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
+    uint32_t k[Q], old[Q];
+    bool hit[Q];
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      k[q] = i < n ? batch_key(eb, pre, i) : 0u;
+    }
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      old[q] = 1u;   // neither transition
+      if (i < n) old[q] = START ? atomicAdd(rcw + k[q], 1u) : atomicSub(rcw + k[q], 1u);
+    }
+#pragma unroll
+    for (int q = 0; q < Q; ++q) {
+      const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      if (START) {
+        hit[q] = i < n && old[q] == 0u;
+        if (i < n && old[q] >= 65535u) set_error(s.st, ERR_REFCOUNT);
+      } else {
+        hit[q] = i < n && old[q] == 1u;
+        if (i < n && old[q] == 0u) {   // more closings than openings: undo, report
+          atomicAdd(rcw + k[q], 1u);
+          set_error(s.st, ERR_REFCOUNT);
+        }
+      }
+    }
+    // a key whose replica was never created (capacity exhausted) has nothing to destroy
+    if (!START) {
+#pragma unroll
+      for (int q = 0; q < Q; ++q)
+        if (hit[q]) hit[q] = mapw[k[q]] >= 0;
+    }
+    uint32_t c = 0, unused = 0, total, t2;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) c += hit[q] ? 1u : 0u;
+    block_exclusive_scan2(c, unused, total, t2);
+    if (threadIdx.x == 0) base_s = total ? atomicAdd(counter, total) : 0u;
+    __syncthreads();
+    c += base_s;
+#pragma unroll
+    for (int q = 0; q < Q; ++q)
+      if (hit[q]) out_list[c++] = k[q];
+    __syncthreads();
+  }
+}
+
+// evict: main[k] += acc[slot]; the freed slot goes on the stack at
+// free_top + i (every listed key holds a replica), so no list atomics are
+// needed.  R keys per row group at a time: list entries, slots, then the
+// pending rows, each as one round of independent loads.
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s, uint32_t w,
+                                                                       const uint32_t* __restrict__ list) {
+  constexpr int R = 4 / C > 0 ? 4 / C : 1;
+  const int lane = threadIdx.x & (G - 1);
+  const uint32_t D4 = s.D >> 2;
+  const uint32_t n = s.st->n_evict;
+  const int32_t top = s.st->free_top;
+  int32_t* mapw = s.map + (uint64_t)w * s.K;
+  float4* main4 = reinterpret_cast<float4*>(s.main);
+  const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const uint64_t step = ng * R;
+  // software-pipelined: a round loads the pending rows of its keys, the
+  // slots of the next round's keys and the list entries of the round after
+  auto load_keys = [&](uint64_t i0, uint32_t (&k)[R]) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) k[r] = i0 + r < n ? list[i0 + r] : 0u;
+  };
+  auto load_slots = [&](uint64_t i0, const uint32_t (&k)[R], int32_t (&sl)[R]) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? mapw[k[r]] : 0;
+  };
+  uint32_t k[R], k1[R];
+  int32_t sl[R];
+  load_keys(g * R, k);
+  load_keys(g * R + step, k1);
+  load_slots(g * R, k, sl);
+  for (uint64_t i0 = g * R; i0 < n; i0 += step) {
+    float4 ac[R][C];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        ac[r][c] = (i0 + r < n && col < D4) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
+      }
+    int32_t sl1[R];
+    uint32_t k2[R];
+    load_slots(i0 + step, k1, sl1);
+    load_keys(i0 + 2 * step, k2);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (i0 + r >= n) break;
+      // each listed key is evicted once, so main[k] has no other writer
+      // here: a vector atomic add gives main + acc without loading main
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) atomicAdd(main4 + (uint64_t)k[r] * D4 + col, ac[r][c]);
+      }
+      if (lane == 0) {
+        mapw[k[r]] = -1;
+        atomicAnd(s.holders + k[r], ~(1u << w));
+        s.slot_owner[sl[r]] = kEmptySlot;
+        s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      k[r] = k1[r];
+      sl[r] = sl1[r];
+      k1[r] = k2[r];
+    }
+  }
+}
+
+// Single thread: account the evictions, then reserve the creations.  The
+// stack initially holds slots S-1 .. 0 (slot 0 on top) and positions below
+// S - high_water are never written, so popping down to alloc_base has used
+// every slot below S - alloc_base.
+__global__ void alloc_kernel(DevState* st, int32_t S) {
+  const uint32_t ne = st->n_evict;
+  st->free_top += (int32_t)ne;
+  st->live -= (int32_t)ne;
+  st->destroyed += ne;
+  const uint32_t n = st->n_create;
+  if ((int64_t)n > (int64_t)st->free_top) {
+    st->errors |= ERR_NO_SLOTS;
+    st->n_create_ok = 0;
+    st->alloc_base = st->free_top;
+    return;
+  }
+  st->alloc_base = st->free_top - (int32_t)n;
+  st->free_top = st->alloc_base;
+  st->n_create_ok = n;
+  st->live += (int32_t)n;
+  st->created += n;
+  if (S - st->alloc_base > st->high_water) st->high_water = S - st->alloc_base;
+}
+
+// create: val = main[k], acc = 0, take a slot from the stack (R keys per
+// row group at a time, as in evict_kernel)
+template <int G, int C>
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store s, uint32_t w,
+                                                                        const uint32_t* __restrict__ list) {
+  constexpr int R = 4 / C > 0 ? 4 / C : 1;
+  const int lane = threadIdx.x & (G - 1);
+  const uint32_t D4 = s.D >> 2;
+  const uint32_t n = s.st->n_create_ok;
+  const int32_t base = s.st->alloc_base;
+  int32_t* mapw = s.map + (uint64_t)w * s.K;
+  const float4* main4 = reinterpret_cast<const float4*>(s.main);
+  float4* val4 = reinterpret_cast<float4*>(s.val);
+  float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const uint64_t step = ng * R;
+  // software-pipelined: a round loads the main rows of its keys and the list
+  // entries and slots of the next round together
+  auto load_entries = [&](uint64_t i0, uint32_t (&k)[R], int32_t (&sl)[R]) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const bool v = i0 + r < n;
+      k[r] = v ? list[i0 + r] : 0u;
+      // slots popped from the top of the stack: lowest free slots come first
+      sl[r] = v ? s.free_stack[base + (int32_t)(n - 1 - (i0 + r))] : 0;
+    }
+  };
+  uint32_t k[R];
+  int32_t sl[R];
+  load_entries(g * R, k, sl);
+  for (uint64_t i0 = g * R; i0 < n; i0 += step) {
+    float4 m[R][C];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        m[r][c] = (i0 + r < n && col < D4) ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
+      }
+    uint32_t k1[R];
+    int32_t sl1[R];
+    load_entries(i0 + step, k1, sl1);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (i0 + r >= n) break;
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) {
+          val4[(uint64_t)sl[r] * D4 + col] = m[r][c];
+          acc4[(uint64_t)sl[r] * D4 + col] = f4zero();
+        }
+      }
+      if (lane == 0) {
+        mapw[k[r]] = sl[r];
+        atomicOr(s.holders + k[r], 1u << w);
+        s.slot_owner[sl[r]] = ((unsigned long long)w << 32) | k[r];
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      k[r] = k1[r];
+      sl[r] = sl1[r];
+    }
+  }
+}
+
+}  // namespace
+
+void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint32_t tag, uint32_t* out,
+                         uint32_t* count, int sms, cudaStream_t stream) {
+  if (n == 0) return;
+  uint64_t b = (n + kDedupTile - 1) / kDedupTile;
+  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+  note_launches(1);
+  intent_dedup_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, keys, n, tag, out, count);
+}
+
+void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
+                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
+  // all opening lists first, then all closing lists, in batches of kEventLists
+  const uint64_t cap_blocks = (uint64_t)sms * 8;
+  for (int pass = 0; pass < 2; ++pass) {
+    const int sign = pass == 0 ? +1 : -1;
+    EventBatch eb{};
+    uint64_t cap = 0;
+    auto flush = [&]() {
+      if (eb.n == 0) return;
+      uint64_t b = (cap + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
+      if (b > cap_blocks) b = cap_blocks;
+      if (b == 0) b = 1;
+      note_launches(1);
+      if (pass == 0)
+        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list);
+      else
+        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, evict_list);
+      eb = EventBatch{};
+      cap = 0;
+    };
+    for (int i = 0; i < nlists; ++i) {
+      if (lists[i].sign != sign) continue;
+      eb.keys[eb.n] = lists[i].keys;
+      eb.count[eb.n] = lists[i].count;
+      eb.n += 1;
+      cap += lists[i].cap;   // the kernel covers the batch's lists as one index space
+      if (eb.n == kEventLists) flush();
+    }
+    flush();
+  }
+}
+
+void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
+                         const uint32_t* evict_list, uint64_t max_events, int sms,
+                         cudaStream_t stream) {
+  dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
+    constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
+    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // keys per group, as in the kernels
+    const unsigned grid = grid_for((max_events + R - 1) / R, G, sms);
+    note_launches(3);
+    evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list);
+    alloc_kernel<<<1, 1, 0, stream>>>(s.st, (int32_t)s.S);
+    create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, create_list);
+  });
+}
+
+}  // namespace adapm

@@ -1,4 +1,4 @@
-// Host-side launchers of the store kernels (store.cu) and step kernels (steps.cu).
+// Host-side launchers of the kernels in store.cu, push.cu and advance.cu, and of the step kernels (steps.cu).
 #pragma once
 
 #include "internal.cuh"
