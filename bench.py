@@ -541,16 +541,21 @@ WORKLOADS = {"micro": Micro, "mf": MF, "tiny_mf": TinyMF, "complex": ComplEx, "s
 # ---------------------------------------------------------------------------
 # algorithmic bytes: the minimum each operation must move (keys 4 B, row D*4 B)
 # ---------------------------------------------------------------------------
-def alg_bytes_per_step(wk, d, steps):
-    """d: differences of the library counters over `steps` profiled steps."""
+def alg_bytes_per_step(wk, d, steps, relocate=False):
+    """d: differences of the library counters over `steps` profiled steps.
+
+    A distinct pushed key costs 4 rows when its target is a replica (value and pending updates, read and
+    written) and 2 when it is main.  Always replicating, every key a worker pushes has a replica; with
+    relocation the split is not counted, so every target is taken as main (a lower bound)."""
     row = wk.row
     per = {k: v / steps for k, v in d.items()}
     R, U = per["push_rows"], per["push_unique"]
+    tgt = 2 * row if relocate else 4 * row
     out = {
         # read keys + scatter rows, and one row read per distinct key (+ its slot)
-        "push": R * (4 + row) + U * (4 + 4 * row),
+        "push": R * (4 + row) + U * (4 + tgt),
         # the scatter kernel alone also reads the sorted (key, position) pairs
-        "push_kernel": R * (8 + row) + U * (4 + 4 * row),
+        "push_kernel": R * (8 + row) + U * (4 + tgt),
         # main += pending (2 rows per key); val := main, pending := 0 (3 rows per replica)
         "sync": per["sync_keys"] * 2 * row + per["sync_replicas"] * 3 * row,
         # destroy: read pending, read+write main; create: read main, write val and pending
@@ -567,7 +572,7 @@ def alg_bytes_per_step(wk, d, steps):
     return out
 
 
-COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "created", "destroyed")
+COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "created", "destroyed", "relocations")
 
 
 def run_ours(args, ws, rank, local):
@@ -579,7 +584,8 @@ def run_ours(args, ws, rank, local):
     t0 = time.time()
     wk.prepare(total_clocks + 2 * args.steps + 2)
     init = wk.init_store()
-    pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init)
+    pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
+                                relocate=args.relocate)
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -642,7 +648,8 @@ def run_ours(args, ws, rank, local):
     peak, peak_src = load_peaks()
 
     steps = args.steps
-    alg = alg_bytes_per_step(wk, {k: s1[k] - s0[k] for k in COUNTERS}, steps)
+    delta = {k: s1[k] - s0[k] for k in COUNTERS}
+    alg = alg_bytes_per_step(wk, delta, steps, args.relocate)
     ops = {}
     for name, (t_ms, calls) in prof.items():
         if calls == 0:
@@ -679,12 +686,16 @@ def run_ours(args, ws, rank, local):
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "samples_per_s": samples if wk.samples_per_step else None,
         "config": dict(wk.config(), parallelism=f"replicas{ws}",
+                       placement="relocate" if args.relocate else "replicate",
                        l2="inputs larger than L2 (no flush)"),
         "gpu_launches": int(launches),
         "clocks": clk,
         "roofline": roofline,
         "ops": ops,
         "stats": {k: stats[k] for k in ("live_replicas", "high_water", "capacity")},
+        # replica management per step (profiled pass): what relocation saves against always replicating
+        "replica_events_per_step": {k: delta[k] / steps for k in ("created", "destroyed", "sync_replicas",
+                                                                   "sync_keys", "relocations")},
         "setup_s": setup_s,
     }
     if e2e_ms is not None:
@@ -716,7 +727,7 @@ def oracle_sample(workload, budget_s, args):
         touched = np.unique(np.concatenate(list(kmap.values())))
         rel = {k: np.searchsorted(touched, v) for k, v in kmap.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.value_len, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
         g = np.random.default_rng(0)
         deltas = (g.standard_normal((cfg.batch, cfg.value_len)) * cfg.delta_std).astype(np.float32)
 
@@ -749,7 +760,7 @@ def oracle_sample(workload, budget_s, args):
         rel = {k: (np.searchsorted(touched, a), np.searchsorted(touched, b), v)
                for k, (a, b, v) in data.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
 
         def work(w, cl):
             a, b, v = rel[(w, cl)]
@@ -772,7 +783,7 @@ def oracle_sample(workload, budget_s, args):
         data = wl.tiny_mf_dataset(cfg)
         nclk = wl.tiny_mf_clocks(cfg, data[3])
         init = hashgen.init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init)
+        pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=args.relocate)
         bt = {(w, c): [x.numpy() for x in wl.tiny_mf_batch(cfg, data, w, c)]
               for w in range(cfg.workers) for c in range(nclk + cfg.lookahead + 1)}
 
@@ -811,7 +822,7 @@ def oracle_sample(workload, budget_s, args):
         touched = np.unique(np.concatenate([keys_full(b) for b in batches.values()]))
         theta = cfg.theta_dim if workload == "complex" else cfg.dim
         init = hashgen.init_rows_np(touched, cfg.value_len, theta, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
         rel = lambda x: np.searchsorted(touched, x)  # noqa: E731
 
         if workload == "complex":
@@ -895,6 +906,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--relocate", action="store_true",
+                    help="relocate a key to its only worker with active intent instead of always replicating")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -71,12 +71,27 @@ typedef struct {
   uint64_t replica_capacity; /* max live replicas over all workers; 0 = min(W*K, 2^24) */
   const float* init_values;  /* K*D floats (host or device), copied at create; NULL = zeros */
   void* stream;              /* cudaStream_t to run on; NULL = a stream owned by the library */
+  int32_t relocate;          /* 0: replicate every active intent (AdaPM without relocation,
+                                Sec. 5.5); 1: relocate a key to the only worker with active
+                                intent, replicate while several have it (Sec. 4.1, App. B.3) */
 } adapm_config;
 
 /* Create a manager: main store = init_values, every clock 0, no intents, no
- * replicas.  Memory: K*D*4 (main) + W*K*6 (slot map, refcounts) + K*4
- * (holder masks) + K*4 (scratch) + capacity*(2*D*4 + 12) bytes of device
- * memory.  Returns ADAPM_ENOMEM if it does not fit. */
+ * replicas, every key at its home (owned by no worker).  Memory: K*D*4 (main)
+ * + W*K*8 (slot maps, refcounts) + K*8 (holder masks, intent stamps) + K*2
+ * with relocate (owner and active-worker count) + capacity*(2*D*4 + 12)
+ * bytes of device memory.  Returns ADAPM_ENOMEM if it does not fit.
+ *
+ * Relocation (relocate = 1).  Every key has an owner: its home at first,
+ * later the last worker that was the only one with active intent for it.
+ * The owner reads and writes the main copy directly and holds no replica;
+ * every other worker with active intent holds a replica.  Whenever exactly
+ * one worker has active intent for a key and does not own it, the key is
+ * relocated to that worker: a replica it holds is destroyed first (its
+ * pending updates merged into main), then it becomes the owner.  Ownership
+ * stays put when the owner's intent expires while others still have active
+ * intent (Fig. 10a), and while nobody has.  Pull, push and sync are the
+ * same in both modes: a worker without a replica uses the main copy. */
 adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out);
 
 /* Wait for outstanding work and free everything the context owns. */
@@ -97,7 +112,9 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
 /* advanceClock() of `worker` (Sec. 3): C^worker += 1.  Replicas whose last
  * active intent expired are destroyed (their updates merged into main), then
  * replicas for keys whose first intent became active are created (value
- * copied from main).  A key that stays active keeps its replica untouched. */
+ * copied from main).  A key that stays active keeps its replica untouched.
+ * With relocation, keys are relocated as the worker's intents start and end
+ * (see adapm_create); this can destroy another worker's replica. */
 adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker);
 
 /* Read n rows: out[i] = worker's replica of keys[i] if it holds one, else the
@@ -197,6 +214,10 @@ adapm_status adapm_replica_rows(adapm_ctx* ctx, uint32_t worker, const uint32_t*
 adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                              uint32_t* out);
 
+/* Owner of each key (int32 out): the worker that holds the key's main copy,
+ * -1 while it is at its home.  Always -1 without relocation. */
+adapm_status adapm_owners(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, int32_t* out);
+
 /* Rows of the main copy. */
 adapm_status adapm_read_main(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, float* out);
 
@@ -210,6 +231,7 @@ typedef struct {
   uint64_t push_unique;      /* distinct keys per push, summed over pushes */
   uint64_t sync_keys;        /* keys merged by sync, cumulative */
   uint64_t sync_replicas;    /* replicas refreshed by sync, cumulative */
+  uint64_t relocations;      /* owner changes, cumulative (relocation only) */
 } adapm_stats;
 
 adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);

@@ -25,7 +25,7 @@ EXPORTS = [
     "adapm_create", "adapm_destroy", "adapm_intent", "adapm_advance_clock", "adapm_pull",
     "adapm_push", "adapm_sync", "adapm_wait", "adapm_mf_step", "adapm_complex_step",
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
-    "adapm_refcounts", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
+    "adapm_refcounts", "adapm_owners", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
     "adapm_profile_read", "adapm_kernel_launches", "adapm_push_noalloc", "adapm_last_error",
     "adapm_debug_fail_next_barrier",
 ]
@@ -39,6 +39,7 @@ class Config(ctypes.Structure):
         ("replica_capacity", ctypes.c_uint64),
         ("init_values", ctypes.c_void_p),
         ("stream", ctypes.c_void_p),
+        ("relocate", ctypes.c_int32),
     ]
 
 
@@ -54,6 +55,7 @@ class Stats(ctypes.Structure):
         ("push_unique", ctypes.c_uint64),
         ("sync_keys", ctypes.c_uint64),
         ("sync_replicas", ctypes.c_uint64),
+        ("relocations", ctypes.c_uint64),
     ]
 
 
@@ -92,6 +94,7 @@ def load(path=LIB_PATH):
         "adapm_replica_keys": [P, U32, P, U64, ctypes.POINTER(U64)],
         "adapm_replica_rows": [P, U32, P, U64, P, P, P],
         "adapm_refcounts": [P, U32, P, U64, P],
+        "adapm_owners": [P, P, U64, P],
         "adapm_read_main": [P, P, U64, P],
         "adapm_get_stats": [P, ctypes.POINTER(Stats)],
         "adapm_profile_enable": [P, I],
@@ -172,7 +175,7 @@ class ParameterManager:
     """One adapm context.  Device arrays are used in place; host arrays are copied."""
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
-                 stream=None):
+                 stream=None, relocate=False):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -185,8 +188,9 @@ class ParameterManager:
         # torch's default stream has handle 0; the ABI reads NULL as "make a
         # stream of your own", so name the legacy default stream (0x1) instead
         handle = stream.cuda_stream or _CUDA_STREAM_LEGACY
+        self.relocate = bool(relocate)
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
-                     ctypes.c_void_p(handle))
+                     ctypes.c_void_p(handle), int(self.relocate))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:
@@ -315,6 +319,13 @@ class ParameterManager:
         out = np.zeros(k.n, np.uint32)
         self._check(self._lib.adapm_refcounts(self._h, worker, k.ptr, k.n, _out_ptr(out)))
         return out.astype(np.int64)
+
+    def owners(self, keys):
+        """Owner worker of each key, -1 while it is at its home."""
+        k = _keys(keys)
+        out = np.zeros(k.n, np.int32)
+        self._check(self._lib.adapm_owners(self._h, k.ptr, k.n, _out_ptr(out)))
+        return out
 
     def read_main(self, keys):
         k = _keys(keys)

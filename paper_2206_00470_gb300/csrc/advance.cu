@@ -111,15 +111,28 @@ __device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32
   return eb.keys[l][i - pre[l]];
 }
 
-// Refcount transitions of one advance.  All lists whose window opens are
-// applied first (START, rc += 1; a key whose count was 0 is listed for
-// creation), then all lists whose window closes (rc -= 1; a key whose count
-// reaches 0 and that holds a replica is listed for eviction).  Every key of a
-// closing list had a positive count before the advance (its intent was
-// active), so with the openings first a key in both kinds of list never
-// crosses 0, and one atomic per listed key gives exactly the transitions of
-// the net change.  Four keys per thread and round; one list append per block
-// and round.  The order of a list is not specified.
+// Refcount transitions of one advance of worker w.  All lists whose window
+// opens are applied first (START, rc += 1), then all lists whose window
+// closes (rc -= 1).  Every key of a closing list had a positive count before
+// the advance (its intent was active), so with the openings first a key in
+// both kinds of list never crosses 0, and one atomic per listed key gives
+// exactly the transitions of the net change: 0 -> 1 (w's intent for k became
+// active, a "join") and 1 -> 0 (a "leave").  Only the thread that sees a
+// key's transition handles it, so the per-key state below has one writer.
+//
+// Always replicate: a join lists k for creation; a leave lists w's replica
+// slot (if it got one) for eviction.
+// Relocation (Sec. 4.1, App. B.3): own[k] counts the workers with active
+// intent and names the owner, which holds no replica.  A join with no other
+// worker active makes w the owner; otherwise w gets a replica unless it
+// owns k already.  A leave destroys w's replica (if any); when exactly one
+// worker stays active and it holds a replica (so it is not the owner), that
+// replica is destroyed too and the worker becomes the owner.  The holders
+// other than w come from holders[k], which only w's own advance changes.
+//
+// The create list takes keys (of worker w), the evict list slots (of any
+// worker).  Four keys per thread and round; one list append per block and
+// round.  The order of a list is not specified.
 template <bool START>
 __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list) {
   if (sort_failed(s.st)) return;
@@ -128,12 +141,13 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
   uint32_t* rcw = s.rc + (uint64_t)w * s.K;
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
   uint32_t* counter = START ? &s.st->n_create : &s.st->n_evict;
+  const bool reloc = s.own != nullptr;
   uint32_t pre[kEventLists + 1];
   const uint32_t n = batch_prefix(eb, pre);
   const uint32_t stride = gridDim.x * blockDim.x * Q;
   for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
-    uint32_t k[Q], old[Q];
-    bool hit[Q];
+    uint32_t k[Q], old[Q], e0[Q], e1[Q];
+    bool hit[Q], hit1[Q];
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
       const uint32_t i = b + q * blockDim.x + threadIdx.x;
@@ -148,6 +162,7 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
       const uint32_t i = b + q * blockDim.x + threadIdx.x;
+      hit1[q] = false;
       if (START) {
         hit[q] = i < n && old[q] == 0u;
         if (i < n && old[q] >= 65535u) set_error(s.st, ERR_REFCOUNT);
@@ -159,94 +174,137 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
         }
       }
     }
-    // a key whose replica was never created (capacity exhausted) has nothing to destroy
-    if (!START) {
+    uint32_t moved = 0;   // owner changes in this round
+    if (START) {
+      // keys with a transition are distinct, so all their loads go first
+      uint32_t o[Q] = {};
 #pragma unroll
       for (int q = 0; q < Q; ++q)
-        if (hit[q]) hit[q] = mapw[k[q]] >= 0;
-    }
-    uint32_t c = 0, unused = 0, total, t2;
+        if (reloc && hit[q]) o[q] = s.own[k[q]];
 #pragma unroll
-    for (int q = 0; q < Q; ++q) c += hit[q] ? 1u : 0u;
-    block_exclusive_scan2(c, unused, total, t2);
-    if (threadIdx.x == 0) base_s = total ? atomicAdd(counter, total) : 0u;
+      for (int q = 0; q < Q; ++q) {
+        e0[q] = k[q];
+        if (reloc && hit[q]) {
+          const uint32_t m = own_count(o[q]);
+          const int owner = own_owner(o[q]);
+          if (m == 0u) {   // the only worker with active intent: relocate to w
+            s.own[k[q]] = own_pack((int)w, 1u);
+            moved += owner != (int)w ? 1u : 0u;
+            hit[q] = false;
+          } else {
+            s.own[k[q]] = own_pack(owner, m + 1u);
+            hit[q] = owner != (int)w;
+          }
+        }
+      }
+    } else {
+      int32_t sl[Q];
+      uint32_t o[Q] = {}, hm[Q] = {};
+#pragma unroll
+      for (int q = 0; q < Q; ++q) {
+        sl[q] = hit[q] ? mapw[k[q]] : -1;
+        if (reloc && hit[q]) {
+          o[q] = s.own[k[q]];
+          hm[q] = s.holders[k[q]];
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < Q; ++q) {
+        if (reloc && hit[q]) {
+          const uint32_t m = own_count(o[q]) - 1u;
+          int owner = own_owner(o[q]);
+          const uint32_t rem = hm[q] & ~(1u << w);
+          if (m == 1u && rem != 0u) {   // one worker left, holding a replica: relocate to it
+            const uint32_t a = (uint32_t)(__ffs(rem) - 1);
+            e1[q] = (uint32_t)s.map[(uint64_t)a * s.K + k[q]];
+            hit1[q] = true;
+            owner = (int)a;
+            moved += 1u;
+          }
+          s.own[k[q]] = own_pack(owner, m);
+        }
+        // a key whose replica was never created (capacity exhausted) has nothing to destroy
+        hit[q] = sl[q] >= 0;
+        e0[q] = (uint32_t)sl[q];
+      }
+    }
+    uint32_t c = 0, total, mtotal;
+#pragma unroll
+    for (int q = 0; q < Q; ++q) c += (hit[q] ? 1u : 0u) + (hit1[q] ? 1u : 0u);
+    block_exclusive_scan2(c, moved, total, mtotal);
+    if (threadIdx.x == 0) {
+      base_s = total ? atomicAdd(counter, total) : 0u;
+      if (mtotal) atomicAdd(&s.st->relocations, (unsigned long long)mtotal);
+    }
     __syncthreads();
     c += base_s;
 #pragma unroll
-    for (int q = 0; q < Q; ++q)
-      if (hit[q]) out_list[c++] = k[q];
+    for (int q = 0; q < Q; ++q) {
+      if (hit[q]) out_list[c++] = e0[q];
+      if (hit1[q]) out_list[c++] = e1[q];
+    }
     __syncthreads();
   }
 }
 
-// evict: main[k] += acc[slot]; the freed slot goes on the stack at
-// free_top + i (every listed key holds a replica), so no list atomics are
-// needed.  R keys per row group at a time: list entries, slots, then the
-// pending rows, each as one round of independent loads.
+// evict: main[k] += acc[slot] for every listed slot (any worker's: a
+// relocation in this advance destroys another worker's replica); the freed
+// slot goes on the stack at free_top + i, so no list atomics are needed.  R
+// slots per row group at a time: the slots' owner records and pending rows
+// as one round of independent loads, together with the next round's slots.
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s, uint32_t w,
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s,
                                                                        const uint32_t* __restrict__ list) {
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint32_t n = s.st->n_evict;
   const int32_t top = s.st->free_top;
-  int32_t* mapw = s.map + (uint64_t)w * s.K;
   float4* main4 = reinterpret_cast<float4*>(s.main);
   const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   const uint64_t step = ng * R;
-  // software-pipelined: a round loads the pending rows of its keys, the
-  // slots of the next round's keys and the list entries of the round after
-  auto load_keys = [&](uint64_t i0, uint32_t (&k)[R]) {
+  auto load_slots = [&](uint64_t i0, int32_t (&sl)[R]) {
 #pragma unroll
-    for (int r = 0; r < R; ++r) k[r] = i0 + r < n ? list[i0 + r] : 0u;
+    for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? (int32_t)list[i0 + r] : 0;
   };
-  auto load_slots = [&](uint64_t i0, const uint32_t (&k)[R], int32_t (&sl)[R]) {
-#pragma unroll
-    for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? mapw[k[r]] : 0;
-  };
-  uint32_t k[R], k1[R];
   int32_t sl[R];
-  load_keys(g * R, k);
-  load_keys(g * R + step, k1);
-  load_slots(g * R, k, sl);
+  load_slots(g * R, sl);
   for (uint64_t i0 = g * R; i0 < n; i0 += step) {
+    unsigned long long ow[R];
     float4 ac[R][C];
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+    for (int r = 0; r < R; ++r) {
+      ow[r] = i0 + r < n ? s.slot_owner[sl[r]] : 0ull;
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
         ac[r][c] = (i0 + r < n && col < D4) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
       }
+    }
     int32_t sl1[R];
-    uint32_t k2[R];
-    load_slots(i0 + step, k1, sl1);
-    load_keys(i0 + 2 * step, k2);
+    load_slots(i0 + step, sl1);
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       if (i0 + r >= n) break;
-      // each listed key is evicted once, so main[k] has no other writer
-      // here: a vector atomic add gives main + acc without loading main
+      const uint32_t k = (uint32_t)ow[r], a = (uint32_t)(ow[r] >> 32);
+      // vector atomic adds: main[k] may receive two pending rows in one
+      // launch (the leaving worker's and a relocated holder's), and needs
+      // no load
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        if (col < D4) atomicAdd(main4 + (uint64_t)k[r] * D4 + col, ac[r][c]);
+        if (col < D4) atomicAdd(main4 + (uint64_t)k * D4 + col, ac[r][c]);
       }
       if (lane == 0) {
-        mapw[k[r]] = -1;
-        atomicAnd(s.holders + k[r], ~(1u << w));
+        s.map[(uint64_t)a * s.K + k] = -1;
+        atomicAnd(s.holders + k, ~(1u << a));
         s.slot_owner[sl[r]] = kEmptySlot;
         s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
       }
     }
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-      k[r] = k1[r];
-      sl[r] = sl1[r];
-      k1[r] = k2[r];
-    }
+    for (int r = 0; r < R; ++r) sl[r] = sl1[r];
   }
 }
 
@@ -390,10 +448,10 @@ void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list
                          cudaStream_t stream) {
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // keys per group, as in the kernels
+    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // list entries per group, as in the kernels
     const unsigned grid = grid_for((max_events + R - 1) / R, G, sms);
     note_launches(3);
-    evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list);
+    evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, evict_list);
     alloc_kernel<<<1, 1, 0, stream>>>(s.st, (int32_t)s.S);
     create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, create_list);
   });

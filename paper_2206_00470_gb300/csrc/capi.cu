@@ -213,11 +213,13 @@ adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventLis
   for (const auto& e : ev) total += e.cap;
   if (total == 0) return ADAPM_OK;
   uint32_t *create_list = nullptr, *evict_list = nullptr;
+  // with relocation a leaving key can also destroy another worker's replica
+  const uint64_t max_events = ctx->s.own ? 2 * total : total;
   CK(pool_alloc(ctx, &create_list, total));
-  CK(pool_alloc(ctx, &evict_list, total));
+  CK(pool_alloc(ctx, &evict_list, max_events));
   CK(cudaMemsetAsync(&ctx->dstate->n_create, 0, 2 * sizeof(uint32_t), ctx->stream));
   launch_events(ctx->s, w, ev.data(), (int)ev.size(), create_list, evict_list, ctx->sms, ctx->stream);
-  launch_evict_create(ctx->s, w, create_list, evict_list, total, ctx->sms, ctx->stream);
+  launch_evict_create(ctx->s, w, create_list, evict_list, max_events, ctx->sms, ctx->stream);
   pool_free(ctx, create_list);
   pool_free(ctx, evict_list);
   return check_launch(ctx, "apply_events");
@@ -295,7 +297,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   *out = nullptr;
   if (cfg->num_keys < 1 || cfg->num_keys >= 0xFFFFFFFFull || cfg->value_len == 0 ||
       cfg->value_len % 4 != 0 || cfg->value_len > 1024 || cfg->num_workers < 1 ||
-      cfg->num_workers > (uint32_t)kMaxWorkers)
+      cfg->num_workers > (uint32_t)kMaxWorkers || (cfg->relocate != 0 && cfg->relocate != 1))
     return ADAPM_EINVAL;
   adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
   if (!ctx) return ADAPM_ENOMEM;
@@ -335,7 +337,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       !dmalloc((void**)&s.acc, S * D * 4) || !dmalloc((void**)&s.map, W * K * 4) ||
       !dmalloc((void**)&s.rc, W * K * 4) || !dmalloc((void**)&s.holders, K * 4) ||
       !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
-      !dmalloc((void**)&s.stamp, K * 4) ||
+      !dmalloc((void**)&s.stamp, K * 4) || (cfg->relocate && !dmalloc((void**)&s.own, K * 2)) ||
       !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
     cudaGetLastError();
     return bail(ADAPM_ENOMEM);
@@ -352,6 +354,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   ok &= cudaMemsetAsync(s.rc, 0, W * K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.holders, 0, K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.stamp, 0, K * 4, st) == cudaSuccess;   // intent tags start at 1
+  if (s.own) ok &= cudaMemsetAsync(s.own, 0, K * 2, st) == cudaSuccess;   // home, no active worker
   DevState h{};
   h.free_top = (int32_t)S;
   ok &= cudaMemcpyAsync(ctx->dstate, &h, sizeof h, cudaMemcpyHostToDevice, st) == cudaSuccess;
@@ -370,7 +373,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
-                  s.stamp, ctx->dstate};
+                  s.stamp, s.own, ctx->dstate};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& t : ctx->pending) {
@@ -764,6 +767,22 @@ adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* ke
   return check_launch(ctx, "refcounts");
 }
 
+adapm_status adapm_owners(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, int32_t* out) {
+  adapm_status st = check_ctx(ctx);
+  if (st != ADAPM_OK) return st;
+  if (n > kMaxN || (n > 0 && (!keys || !out))) return fail(ctx, ADAPM_EINVAL, "bad arguments");
+  if (n == 0) return ADAPM_OK;
+  Input<uint32_t> in;
+  CK(stage_in(ctx, keys, n, &in));
+  Output<int32_t> o;
+  CK(stage_out(ctx, out, n, &o));
+  launch_owners(ctx->s, in.dev, n, o.dev, ctx->stream);
+  CK(finish_out(ctx, &o));
+  pool_free(ctx, in.owned);
+  CK(cudaStreamSynchronize(ctx->stream));
+  return check_launch(ctx, "owners");
+}
+
 adapm_status adapm_read_main(adapm_ctx* ctx, const uint32_t* keys, uint64_t n, float* out) {
   adapm_status st = check_ctx(ctx);
   if (st != ADAPM_OK) return st;
@@ -797,6 +816,7 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
   out->push_unique = h.push_unique;
   out->sync_keys = h.sync_keys;
   out->sync_replicas = h.sync_replicas;
+  out->relocations = h.relocations;
   return ADAPM_OK;
 }
 

@@ -9,6 +9,9 @@
 //   slot_owner  [S]    uint64   (w << 32) | k of a live slot, kEmptySlot if free
 //   free_stack  [S]    int32    free slots, top at free_stack[free_top - 1]
 //   stamp       [K]    uint32   tag of the last Intent call that listed k
+//   own         [K]    uint16   relocation mode only: ((owner + 1) << 8) |
+//                               number of workers with active intent; owner
+//                               -1 is the key's home (no worker held it yet)
 //   DevState                    counters and the sticky error bits
 #pragma once
 
@@ -35,7 +38,7 @@ struct DevState {
   int32_t free_top;       // free slots on the stack
   int32_t high_water;     // slots [0, high_water) have been used
   uint32_t n_create;      // keys appended to the create list of this advance
-  uint32_t n_evict;       // keys appended to the evict list of this advance
+  uint32_t n_evict;       // slots appended to the evict list of this advance
   int32_t alloc_base;     // first stack index popped by this advance
   uint32_t n_create_ok;   // creates that got a slot
   uint32_t errors;        // ErrBits, sticky until read by adapm_wait
@@ -48,6 +51,7 @@ struct DevState {
   unsigned long long push_unique;     // distinct keys over all pushes (cumulative)
   unsigned long long sync_keys;       // keys merged by sync (cumulative)
   unsigned long long sync_replicas;   // replicas refreshed by sync (cumulative)
+  unsigned long long relocations;     // owner changes (relocation mode, cumulative)
   // grid barriers of the sort: blocks arrived, over the context's lifetime
   // (a line of its own, away from the counters above)
   alignas(128) unsigned long long bar_arrivals;
@@ -64,12 +68,20 @@ struct Store {
   unsigned long long* slot_owner;
   int32_t* free_stack;
   uint32_t* stamp;
+  uint16_t* own;   // null unless relocation mode
   DevState* st;
   uint64_t K;
   uint64_t S;
   uint32_t D;
   uint32_t W;
 };
+
+// Fields of own[k] (relocation mode).
+__device__ __forceinline__ uint32_t own_count(uint32_t o) { return o & 0xFFu; }
+__device__ __forceinline__ int own_owner(uint32_t o) { return (int)(o >> 8) - 1; }
+__device__ __forceinline__ uint16_t own_pack(int owner, uint32_t count) {
+  return (uint16_t)(((uint32_t)(owner + 1) << 8) | count);
+}
 
 __device__ __forceinline__ void set_error(DevState* st, uint32_t bits) {
   atomicOr(&st->errors, bits);

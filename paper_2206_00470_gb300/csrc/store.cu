@@ -231,6 +231,19 @@ __global__ void refcounts_kernel(Store s, uint32_t w, const uint32_t* __restrict
   }
 }
 
+// owner of each key: -1 at its home (and always without relocation)
+__global__ void owners_kernel(Store s, const uint32_t* __restrict__ keys, uint64_t n, int32_t* __restrict__ out) {
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t k = keys[i];
+    if (k < s.K) out[i] = s.own ? own_owner(s.own[k]) : -1;
+    else {
+      out[i] = -1;
+      set_error(s.st, ERR_KEY_RANGE);
+    }
+  }
+}
+
 __global__ void replica_rows_kernel(Store s, uint32_t w, const uint32_t* __restrict__ keys, uint64_t n,
                                     float* __restrict__ val_out, float* __restrict__ acc_out,
                                     uint8_t* __restrict__ has_out) {
@@ -289,6 +302,13 @@ void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t
   note_launches(1);
   refcounts_kernel<<<(unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, stream>>>(
       s, w, keys, n, out);
+}
+
+void launch_owners(const Store& s, const uint32_t* keys, uint64_t n, int32_t* out, cudaStream_t stream) {
+  if (n == 0) return;
+  note_launches(1);
+  owners_kernel<<<(unsigned)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, stream>>>(s, keys, n,
+                                                                                                 out);
 }
 
 void launch_replica_rows(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, float* val,

@@ -48,6 +48,13 @@ void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint3
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream);
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream);
+// Refcount events of one advance of worker w: keys to create a replica of
+// for w go to create_list, replica slots to destroy (of w, and in relocation
+// mode of a worker the key is relocated to) to evict_list; the counters
+// n_create / n_evict in DevState must be zero.  With cap = the summed caps of
+// the lists, create_list needs cap entries and evict_list cap (always
+// replicate) or 2 * cap (relocation).  launch_evict_create applies both
+// lists; max_events bounds either list's length.
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
                    uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream);
 void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
@@ -56,6 +63,7 @@ void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list
 void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stream);
 void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, uint32_t* out,
                       cudaStream_t stream);
+void launch_owners(const Store& s, const uint32_t* keys, uint64_t n, int32_t* out, cudaStream_t stream);
 void launch_replica_rows(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, float* val,
                          float* acc, uint8_t* has, cudaStream_t stream);
 void launch_init_pool(int32_t* free_stack, uint64_t S, unsigned long long* owner, cudaStream_t stream);

@@ -1,7 +1,8 @@
 """Parity at the full sizes of the workloads, in the bench's launch configuration.
 
 * microbench (100M keys x 64, W=8, 2^20 Zipf(1.1) keys per worker per clock,
-  intent span 2): the manager's semantics are separable by key, so the oracle
+  intent span 2), always replicating and with relocation (owners compared
+  too): the manager's semantics are separable by key, so the oracle
   replays the whole call sequence restricted to a sample of keys (the hottest
   keys of the batches, random batch keys and keys never touched) and every
   value the GPU holds for those keys is compared bit-exactly (dyadic initial
@@ -30,7 +31,8 @@ def dev(x):
     return torch.as_tensor(np.asarray(x), device="cuda")
 
 
-def test_micro_full_size_sampled_keys_bit_exact(gpu_lib):
+@pytest.mark.parametrize("relocate", [False, True])
+def test_micro_full_size_sampled_keys_bit_exact(gpu_lib, relocate):
     cfg = dataclasses.replace(wl.MICRO, span=2)
     K, D, W, B = cfg.num_keys, cfg.value_len, cfg.workers, cfg.batch
     nclk = 3
@@ -38,7 +40,8 @@ def test_micro_full_size_sampled_keys_bit_exact(gpu_lib):
     deltas = {(w, c): wl.micro_deltas(cfg, w, c, B, dyadic=True).numpy() for w in range(W) for c in range(nclk)}
     # the store: dyadic values from the counter hash, generated on the GPU
     init = hashgen.init_store_torch(K, D, D, cfg.seed, 0.0, "cuda", kind="dyadic", chunk_rows=1 << 22)
-    pm = gpu_lib.ParameterManager(K, D, W, replica_capacity=W * (cfg.span + 1) * B, init_values=init)
+    pm = gpu_lib.ParameterManager(K, D, W, replica_capacity=W * (cfg.span + 1) * B, init_values=init,
+                                  relocate=relocate)
     del init
     torch.cuda.empty_cache()
     pulled = {}
@@ -68,7 +71,8 @@ def test_micro_full_size_sampled_keys_bit_exact(gpu_lib):
     pm.wait()
 
     ref = ParameterManagerOracle(sample.size, D, W,
-                                 hashgen.init_rows_np(sample, D, D, cfg.seed, 0.0, kind="dyadic"))
+                                 hashgen.init_rows_np(sample, D, D, cfg.seed, 0.0, kind="dyadic"),
+                                 relocation=relocate)
 
     def restrict(w, c):
         m = masks[(w, c)]
@@ -91,6 +95,7 @@ def test_micro_full_size_sampled_keys_bit_exact(gpu_lib):
         assert np.array_equal(np.nonzero(has)[0], rk)
         assert np.array_equal(val[rk], rval) and np.array_equal(acc[rk], racc)
         assert np.array_equal(pm.refcounts(w, sample), ref.refcounts(w, np.arange(sample.size)))
+    assert np.array_equal(pm.owners(sample), ref.owners(np.arange(sample.size)))
     pm.close()
 
 
