@@ -73,7 +73,7 @@ typedef struct {
   void* stream;              /* cudaStream_t to run on; NULL = a stream owned by the library */
   int32_t relocate;          /* 0: replicate every active intent (AdaPM without relocation,
                                 Sec. 5.5); 1: relocate a key to the only worker with active
-                                intent, replicate while several have it (Sec. 4.1, App. B.3) */
+                                intent, replicate while several have it (Sec. 4.1, App. B.2.4) */
 } adapm_config;
 
 /* Create a manager: main store = init_values, every clock 0, no intents, no

@@ -9,7 +9,9 @@ input generators in synth/, which hold none of the method's arithmetic.
 Modules
   store  intent windows, replica lifetime, pull, push, sync (Sec. 3, Sec. 4.1,
          App. B.1.2, Sec. 5.1 consistency model); optionally the relocation
-         rule of Sec. 4.1 / App. B.3
+         rule of Sec. 4.1 / App. B.2.4
+  timing adaptive action timing (Sec. 4.2, Algorithm 1): the Poisson quantile
+         and the per-worker rate estimate
   steps  the three training steps (App. C: MF, ComplEx KGE, skip-gram WV)
   driver the per-clock loop of a data-parallel worker (Fig. 2 pattern)
 
@@ -21,6 +23,8 @@ Pins (tests/test_oracle_*.py): brute-force active sets from the raw call log,
 the sum invariant with dyadic deltas (bit-exact), hand-worked scenarios in
 tests/golden/, the owner and replica intervals of the paper's Fig. 4b-d and
 Fig. 10a, the owner recomputed by brute force from the call log, the
+Poisson quantile against scipy's, the rate estimate against the closed form
+of its recursion, the
 single-worker reduction to textbook mini-batch SGD,
 fp64 finite-difference gradients, ComplEx scores by complex arithmetic and
 closed forms, Zipf frequencies by chi-square.  No function here is "parity

@@ -37,7 +37,15 @@ Definitions
     acc = 0 (App. B.1.2: the owner merges the updates and propagates them to
     the replica holders; sending only unseen versions gives the same values).
 
-Relocation (Sec. 4.1 and App. B.3, "relocate only when exactly one node has
+Action timing (Sec. 4.2).  action_timing="start" (default) acts on an intent
+exactly when it becomes active.  "signal" acts when the intent is signalled
+(the paper's immediate-action ablation, Sec. 5.8): its window is treated as
+starting at the signalling clock.  "adaptive" follows Algorithm 1
+(oracle/timing.py): every sync is a communication round; after its merge,
+each worker's intents that Algorithm 1 selects are treated as active from
+that round on; an intent no round selected becomes active at its start.
+
+Relocation (Sec. 4.1 and App. B.2.4, "relocate only when exactly one node has
 active intent"; scenarios of Fig. 4b-d and Fig. 10a)
   * Every key has an owner: a worker slot, or its home (-1) before any
     worker has held it.  The owner accesses the main copy directly and holds
@@ -62,6 +70,8 @@ Arithmetic: every sum runs in fp64 and is rounded to fp32 once when stored.
 """
 import numpy as np
 
+from .timing import RateEstimate
+
 
 class OracleError(ValueError):
     """An argument the parameter manager must reject (bad worker, key out of range)."""
@@ -72,7 +82,8 @@ def _f32(x):
 
 
 class ParameterManagerOracle:
-    def __init__(self, num_keys, value_len, num_workers, init, relocation=False):
+    def __init__(self, num_keys, value_len, num_workers, init, relocation=False, action_timing="start",
+                 timing_alpha=None, timing_p=None, timing_lambda0=None):
         init = np.asarray(init, dtype=np.float32)
         if init.shape != (num_keys, value_len):
             raise OracleError("init must have shape (num_keys, value_len)")
@@ -87,6 +98,12 @@ class ParameterManagerOracle:
         self.active = [set() for _ in range(self.W)]  # A_w(C^w) as of w's last call
         self.owner = np.full(self.K, -1, dtype=np.int64)
         self.created = self.destroyed = self.relocations = 0
+        if action_timing not in ("start", "adaptive", "signal"):
+            raise OracleError("action_timing must be 'start', 'adaptive' or 'signal'")
+        self.action_timing = action_timing
+        kw = {k: v for k, v in (("alpha", timing_alpha), ("p", timing_p), ("lambda0", timing_lambda0))
+              if v is not None}
+        self.rates = [RateEstimate(**kw) for _ in range(self.W)]
 
     # -- argument checks ---------------------------------------------------
     def _check_worker(self, w):
@@ -172,6 +189,8 @@ class ParameterManagerOracle:
         start, end = int(start), int(end)
         if end <= start or end <= self.clock[w]:
             return                      # empty or already expired window: nothing to do
+        if self.action_timing == "signal":
+            start = min(start, self.clock[w])   # act as soon as the intent is signalled
         self.intents[w].append((frozenset(int(k) for k in keys), start, end))
         self._reconcile(w)              # activates now if start <= C^w
 
@@ -218,6 +237,25 @@ class ParameterManagerOracle:
             self.main[k] = _f32(total)
             for w in holders:
                 self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+        if self.action_timing == "adaptive":
+            self._act_in_round()
+
+    def _act_in_round(self):
+        """A communication round (one sync) acts on the intents Algorithm 1 selects, worker by worker.
+
+        After the merge (App. B.2.2: the owner merges the updates, then answers the intent signals), every
+        recorded intent of worker w that is not active yet and starts before C^w + b_w is treated as active
+        from now on; intents no round selected still become active at their start clock."""
+        for w in range(self.W):
+            c = self.clock[w]
+            bound = self.rates[w].round(c)
+            acted = False
+            for i, (keys, s, e) in enumerate(self.intents[w]):
+                if c < s < c + bound:
+                    self.intents[w][i] = (keys, c, e)
+                    acted = True
+            if acted:
+                self._reconcile(w)
 
     # -- inspection --------------------------------------------------------------
     def replica_keys(self, w):

@@ -122,7 +122,7 @@ __device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32
 //
 // Always replicate: a join lists k for creation; a leave lists w's replica
 // slot (if it got one) for eviction.
-// Relocation (Sec. 4.1, App. B.3): own[k] counts the workers with active
+// Relocation (Sec. 4.1, App. B.2.4): own[k] counts the workers with active
 // intent and names the owner, which holds no replica.  A join with no other
 // worker active makes w the owner; otherwise w gets a replica unless it
 // owns k already.  A leave destroys w's replica (if any); when exactly one

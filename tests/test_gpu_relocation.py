@@ -1,4 +1,4 @@
-"""GPU parity of the relocation mode (Sec. 4.1, App. B.3) against the CPU oracle.
+"""GPU parity of the relocation mode (Sec. 4.1, App. B.2.4) against the CPU oracle.
 
 The CUDA path runs with relocate=1 through the C ABI and the oracle with relocation=True on the same
 seeded call sequences.  Bit-exact: owners, replica key sets, refcounts, pulled rows and, with dyadic

@@ -1,4 +1,4 @@
-"""Pins of the oracle's relocation mode (Sec. 4.1, App. B.3) against things other than itself.
+"""Pins of the oracle's relocation mode (Sec. 4.1, App. B.2.4) against things other than itself.
 
 * the intent scenarios of Fig. 4b-d and Fig. 10a (tests/golden/relocation_figures.json): the owner and the
   replica intervals that the paper draws, at every clock;
