@@ -585,7 +585,7 @@ def run_ours(args, ws, rank, local):
     wk.prepare(total_clocks + 2 * args.steps + 2)
     init = wk.init_store()
     pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
-                                relocate=args.relocate)
+                                relocate=args.relocate, action_timing=args.timing)
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -687,6 +687,7 @@ def run_ours(args, ws, rank, local):
         "samples_per_s": samples if wk.samples_per_step else None,
         "config": dict(wk.config(), parallelism=f"replicas{ws}",
                        placement="relocate" if args.relocate else "replicate",
+                       action_timing=args.timing,
                        l2="inputs larger than L2 (no flush)"),
         "gpu_launches": int(launches),
         "clocks": clk,
@@ -727,7 +728,8 @@ def oracle_sample(workload, budget_s, args):
         touched = np.unique(np.concatenate(list(kmap.values())))
         rel = {k: np.searchsorted(touched, v) for k, v in kmap.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.value_len, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
+                                    action_timing=args.timing)
         g = np.random.default_rng(0)
         deltas = (g.standard_normal((cfg.batch, cfg.value_len)) * cfg.delta_std).astype(np.float32)
 
@@ -760,7 +762,8 @@ def oracle_sample(workload, budget_s, args):
         rel = {k: (np.searchsorted(touched, a), np.searchsorted(touched, b), v)
                for k, (a, b, v) in data.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
+                                    action_timing=args.timing)
 
         def work(w, cl):
             a, b, v = rel[(w, cl)]
@@ -783,7 +786,8 @@ def oracle_sample(workload, budget_s, args):
         data = wl.tiny_mf_dataset(cfg)
         nclk = wl.tiny_mf_clocks(cfg, data[3])
         init = hashgen.init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=args.relocate)
+        pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=args.relocate,
+                                    action_timing=args.timing)
         bt = {(w, c): [x.numpy() for x in wl.tiny_mf_batch(cfg, data, w, c)]
               for w in range(cfg.workers) for c in range(nclk + cfg.lookahead + 1)}
 
@@ -822,7 +826,8 @@ def oracle_sample(workload, budget_s, args):
         touched = np.unique(np.concatenate([keys_full(b) for b in batches.values()]))
         theta = cfg.theta_dim if workload == "complex" else cfg.dim
         init = hashgen.init_rows_np(touched, cfg.value_len, theta, cfg.seed, cfg.init_std)
-        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate)
+        pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
+                                    action_timing=args.timing)
         rel = lambda x: np.searchsorted(touched, x)  # noqa: E731
 
         if workload == "complex":
@@ -908,6 +913,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--relocate", action="store_true",
                     help="relocate a key to its only worker with active intent instead of always replicating")
+    ap.add_argument("--timing", default="start", choices=["start", "adaptive", "signal"],
+                    help="act on an intent at its start clock, by Algorithm 1 at each sync, or when signalled")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

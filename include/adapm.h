@@ -74,7 +74,32 @@ typedef struct {
   int32_t relocate;          /* 0: replicate every active intent (AdaPM without relocation,
                                 Sec. 5.5); 1: relocate a key to the only worker with active
                                 intent, replicate while several have it (Sec. 4.1, App. B.2.4) */
+  int32_t action_timing;     /* when the manager acts on an intent: ADAPM_ACT_AT_START (0),
+                                ADAPM_ACT_ADAPTIVE (1) or ADAPM_ACT_ON_SIGNAL (2), below */
+  double timing_alpha;       /* ADAPM_ACT_ADAPTIVE: smoothing factor, 0 = 0.1 */
+  double timing_p;           /* ADAPM_ACT_ADAPTIVE: Poisson quantile, 0 = 0.9999 */
+  double timing_lambda0;     /* ADAPM_ACT_ADAPTIVE: initial clocks per round, 0 = 10 */
 } adapm_config;
+
+/* Action timing (Sec. 4.2).
+ *   ADAPM_ACT_AT_START   act when the intent becomes active (C^w reaches C_start).
+ *   ADAPM_ACT_ON_SIGNAL  act when the intent is signalled: the window is
+ *                        treated as starting at the worker's current clock
+ *                        (the immediate-action variant of Sec. 5.8).
+ *   ADAPM_ACT_ADAPTIVE   Algorithm 1: every adapm_sync is a communication
+ *                        round.  After its merge, for each worker w in
+ *                        ascending order, with Delta = C^w - (C^w at the
+ *                        previous round, 0 at first), the estimate becomes
+ *                        (1 - alpha) est + alpha Delta when Delta > 0, and
+ *                        every recorded intent of w with
+ *                        C^w < C_start < C^w + Q(2 max(est, Delta), p)
+ *                        is treated as active from now on (Q = the Poisson
+ *                        quantile of adapm_poisson_quantile).  An intent no
+ *                        round selected becomes active at C_start.
+ * Acting early only moves the start of an intent's window; its end stays. */
+#define ADAPM_ACT_AT_START 0
+#define ADAPM_ACT_ADAPTIVE 1
+#define ADAPM_ACT_ON_SIGNAL 2
 
 /* Create a manager: main store = init_values, every clock 0, no intents, no
  * replicas, every key at its home (owned by no worker).  Memory: K*D*4 (main)
@@ -156,7 +181,9 @@ adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, const uint32_t*
 
 /* Replica synchronisation (App. B.1.2): for every key with replicas,
  * main += the pending updates of all holders (ascending worker order), then
- * every holder's replica := main and its pending updates := 0. */
+ * every holder's replica := main and its pending updates := 0.  With
+ * ADAPM_ACT_ADAPTIVE this is also a communication round of Algorithm 1
+ * (see adapm_config), which may activate intents early. */
 adapm_status adapm_sync(adapm_ctx* ctx);
 
 /* Block until the stream is idle; return and clear the first sticky device
@@ -213,6 +240,13 @@ adapm_status adapm_replica_rows(adapm_ctx* ctx, uint32_t worker, const uint32_t*
 /* Number of the worker's active intents containing each key (uint32 out). */
 adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                              uint32_t* out);
+
+/* The p quantile of a Poisson distribution with mean lambda: the smallest
+ * integer q >= 0 with P(X <= q) >= p, found by adding P(X = j) =
+ * exp(-lambda + j ln lambda - ln j!) for j = 0, 1, ... in that order (the
+ * rule ADAPM_ACT_ADAPTIVE uses).  Host only; needs no GPU.  ADAPM_EINVAL
+ * unless lambda > 0, 0 < p < 1 and out is not NULL. */
+adapm_status adapm_poisson_quantile(double lambda, double p, int64_t* out);
 
 /* Owner of each key (int32 out): the worker that holds the key's main copy,
  * -1 while it is at its home.  Always -1 without relocation. */

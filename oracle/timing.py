@@ -18,7 +18,8 @@ P(X <= q) >= p.  The paper's settings: alpha = 0.1, p = 0.9999, est_0 = 10.
 
 Arithmetic: fp64.  The quantile adds the probabilities P(X = j) for
 j = 0, 1, ... in that order, each computed as exp(-lam + j ln lam - ln j!),
-until the sum reaches p.
+until the sum reaches p (or j passes lam + 64 sqrt(lam) + 64, which no
+quantile with p < 1 - 1e-12 reaches: a guard against rounding).
 """
 import math
 
@@ -32,11 +33,12 @@ def poisson_quantile(lam, p):
     if not (lam > 0.0) or not (0.0 < p < 1.0):
         raise ValueError("need lam > 0 and 0 < p < 1")
     ln_lam = math.log(lam)
+    qmax = lam + 64.0 * math.sqrt(lam) + 64.0    # far past any quantile with p < 1 - 1e-12
     cdf = 0.0
     q = 0
     while True:
         cdf += math.exp(-lam + q * ln_lam - math.lgamma(q + 1.0))
-        if cdf >= p:
+        if cdf >= p or q >= qmax:
             return q
         q += 1
 

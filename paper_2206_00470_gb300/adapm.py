@@ -25,7 +25,7 @@ EXPORTS = [
     "adapm_create", "adapm_destroy", "adapm_intent", "adapm_advance_clock", "adapm_pull",
     "adapm_push", "adapm_sync", "adapm_wait", "adapm_mf_step", "adapm_complex_step",
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
-    "adapm_refcounts", "adapm_owners", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
+    "adapm_refcounts", "adapm_owners", "adapm_poisson_quantile", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
     "adapm_profile_read", "adapm_kernel_launches", "adapm_push_noalloc", "adapm_last_error",
     "adapm_debug_fail_next_barrier",
 ]
@@ -40,7 +40,14 @@ class Config(ctypes.Structure):
         ("init_values", ctypes.c_void_p),
         ("stream", ctypes.c_void_p),
         ("relocate", ctypes.c_int32),
+        ("action_timing", ctypes.c_int32),
+        ("timing_alpha", ctypes.c_double),
+        ("timing_p", ctypes.c_double),
+        ("timing_lambda0", ctypes.c_double),
     ]
+
+
+ACTION_TIMING = {"start": 0, "adaptive": 1, "signal": 2}
 
 
 class Stats(ctypes.Structure):
@@ -95,6 +102,7 @@ def load(path=LIB_PATH):
         "adapm_replica_rows": [P, U32, P, U64, P, P, P],
         "adapm_refcounts": [P, U32, P, U64, P],
         "adapm_owners": [P, P, U64, P],
+        "adapm_poisson_quantile": [ctypes.c_double, ctypes.c_double, ctypes.POINTER(I64)],
         "adapm_read_main": [P, P, U64, P],
         "adapm_get_stats": [P, ctypes.POINTER(Stats)],
         "adapm_profile_enable": [P, I],
@@ -171,11 +179,21 @@ def _out_ptr(t):
     return t.data_ptr() if t.numel() else None
 
 
+def poisson_quantile(lam, p):
+    """The p quantile of Poisson(lam) as the library's adaptive action timing computes it (host only)."""
+    out = ctypes.c_int64()
+    st = load().adapm_poisson_quantile(float(lam), float(p), ctypes.byref(out))
+    if st != OK:
+        raise AdaPMError(st, "adapm_poisson_quantile: need lam > 0 and 0 < p < 1")
+    return out.value
+
+
 class ParameterManager:
     """One adapm context.  Device arrays are used in place; host arrays are copied."""
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
-                 stream=None, relocate=False):
+                 stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
+                 timing_lambda0=0.0):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -189,8 +207,12 @@ class ParameterManager:
         # stream of your own", so name the legacy default stream (0x1) instead
         handle = stream.cuda_stream or _CUDA_STREAM_LEGACY
         self.relocate = bool(relocate)
+        if action_timing not in ACTION_TIMING:
+            raise ValueError(f"action_timing must be one of {sorted(ACTION_TIMING)}")
+        self.action_timing = action_timing
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
-                     ctypes.c_void_p(handle), int(self.relocate))
+                     ctypes.c_void_p(handle), int(self.relocate), ACTION_TIMING[action_timing],
+                     float(timing_alpha), float(timing_p), float(timing_lambda0))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:

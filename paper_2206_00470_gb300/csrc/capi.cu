@@ -5,7 +5,9 @@
 // stream; scratch comes from a context-owned stream-ordered memory pool.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -37,6 +39,8 @@ struct IntentList {
 
 struct WorkerState {
   int64_t clock = 0;
+  double est = 0.0;          // Algorithm 1: clocks per round, smoothed
+  int64_t round_clock = 0;   // clock at the previous round
   std::map<int64_t, std::vector<int64_t>> starts;   // clock -> lists whose window opens
   std::map<int64_t, std::vector<int64_t>> ends;     // clock -> lists whose window closes
 };
@@ -267,6 +271,50 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   return check_launch(ctx, "push");
 }
 
+// The p quantile of Poisson(lam): P(X = j) added for j = 0, 1, ... in order
+// until the sum reaches p.  The loop ends: the sum tends to 1 > p (a bound on
+// the index guards against rounding for huge lam).
+int64_t poisson_quantile(double lam, double p) {
+  const double ln_lam = std::log(lam);
+  const double qmax = lam + 64.0 * std::sqrt(lam) + 64.0;
+  double cdf = 0.0;
+  int64_t q = 0;
+  for (;; ++q) {
+    const double j = (double)q;
+    cdf += std::exp(-lam + j * ln_lam - std::lgamma(j + 1.0));
+    if (cdf >= p || j >= qmax) return q;
+  }
+}
+
+// One communication round of adaptive action timing (Sec. 4.2, Algorithm 1),
+// after the sync's merge: each worker in ascending order updates its rate
+// estimate and activates the recorded intents that start before its clock
+// plus the Poisson bound.
+adapm_status act_in_round(adapm_ctx* ctx) {
+  const double alpha = ctx->cfg.timing_alpha, p = ctx->cfg.timing_p;
+  for (uint32_t w = 0; w < ctx->s.W; ++w) {
+    WorkerState& ws = ctx->workers[w];
+    const int64_t delta = ws.clock - ws.round_clock;
+    if (delta > 0) ws.est = (1.0 - alpha) * ws.est + alpha * (double)delta;
+    ws.round_clock = ws.clock;
+    const int64_t bound = poisson_quantile(2.0 * std::max(ws.est, (double)delta), p);
+    std::vector<EventList> ev;
+    auto it = ws.starts.begin();
+    while (it != ws.starts.end() && it->first < ws.clock + bound) {
+      for (int64_t id : it->second) {
+        const IntentList& L = ctx->lists[id];
+        ev.push_back(EventList{L.keys, L.count, L.cap, +1});
+      }
+      it = ws.starts.erase(it);
+    }
+    if (!ev.empty()) {
+      const adapm_status st = apply_events(ctx, w, ev);
+      if (st != ADAPM_OK) return st;
+    }
+  }
+  return ADAPM_OK;
+}
+
 }  // namespace
 
 bool adapm::ctx_view(adapm_ctx* ctx, CtxView* out) {
@@ -297,11 +345,17 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   *out = nullptr;
   if (cfg->num_keys < 1 || cfg->num_keys >= 0xFFFFFFFFull || cfg->value_len == 0 ||
       cfg->value_len % 4 != 0 || cfg->value_len > 1024 || cfg->num_workers < 1 ||
-      cfg->num_workers > (uint32_t)kMaxWorkers || (cfg->relocate != 0 && cfg->relocate != 1))
+      cfg->num_workers > (uint32_t)kMaxWorkers || (cfg->relocate != 0 && cfg->relocate != 1) ||
+      cfg->action_timing < ADAPM_ACT_AT_START || cfg->action_timing > ADAPM_ACT_ON_SIGNAL ||
+      !(cfg->timing_alpha >= 0.0 && cfg->timing_alpha <= 1.0) ||
+      !(cfg->timing_p >= 0.0 && cfg->timing_p < 1.0) || !(cfg->timing_lambda0 >= 0.0))
     return ADAPM_EINVAL;
   adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
   if (!ctx) return ADAPM_ENOMEM;
   ctx->cfg = *cfg;
+  if (ctx->cfg.timing_alpha == 0.0) ctx->cfg.timing_alpha = 0.1;
+  if (ctx->cfg.timing_p == 0.0) ctx->cfg.timing_p = 0.9999;
+  if (ctx->cfg.timing_lambda0 == 0.0) ctx->cfg.timing_lambda0 = 10.0;
   const uint64_t K = cfg->num_keys, D = cfg->value_len, W = cfg->num_workers;
   uint64_t S = cfg->replica_capacity;
   if (S == 0) S = W * K < (1ull << 24) ? W * K : (1ull << 24);
@@ -362,6 +416,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   ok &= cudaStreamSynchronize(st) == cudaSuccess;
   if (!ok || cudaGetLastError() != cudaSuccess) return bail(ADAPM_ECUDA);
   ctx->workers.resize(W);
+  for (auto& ws : ctx->workers) ws.est = ctx->cfg.timing_lambda0;
   *out = ctx;
   return ADAPM_OK;
 }
@@ -396,6 +451,8 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   if (n > kMaxN || (n > 0 && !keys)) return fail(ctx, ADAPM_EINVAL, "bad keys/n");
   WorkerState& ws = ctx->workers[worker];
   if (clock_end <= clock_start || clock_end <= ws.clock) return ADAPM_OK;   // never active
+  // acting on signal: the window starts now
+  if (ctx->cfg.action_timing == ADAPM_ACT_ON_SIGNAL && clock_start > ws.clock) clock_start = ws.clock;
   ProfScope ps(ctx, 0);
   IntentList L;
   L.cap = n;
@@ -515,9 +572,20 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
 adapm_status adapm_sync(adapm_ctx* ctx) {
   adapm_status st = check_ctx(ctx);
   if (st != ADAPM_OK) return st;
-  ProfScope ps(ctx, 4);
-  launch_sync(ctx->s, ctx->s.S, ctx->sms, ctx->stream);
-  return check_launch(ctx, "sync");
+  {
+    ProfScope ps(ctx, 4);
+    launch_sync(ctx->s, ctx->s.S, ctx->sms, ctx->stream);
+    st = check_launch(ctx, "sync");
+    if (st != ADAPM_OK) return st;
+  }
+  if (ctx->cfg.action_timing == ADAPM_ACT_ADAPTIVE) return act_in_round(ctx);
+  return ADAPM_OK;
+}
+
+adapm_status adapm_poisson_quantile(double lambda, double p, int64_t* out) {
+  if (!out || !(lambda > 0.0) || !(p > 0.0 && p < 1.0)) return ADAPM_EINVAL;
+  *out = poisson_quantile(lambda, p);
+  return ADAPM_OK;
 }
 
 adapm_status adapm_debug_fail_next_barrier(adapm_ctx* ctx) {

@@ -61,8 +61,26 @@ def test_create_rejects_bad_configs_without_touching_the_gpu(lib_path):
         adapm.Config(10, 4, 0, 0, None, None),         # no workers
         adapm.Config(10, 4, 33, 0, None, None),        # more than 32 workers
         adapm.Config(2 ** 32 - 1, 4, 1, 0, None, None),
+        adapm.Config(10, 4, 1, 0, None, None, 2),                    # relocate is 0 or 1
+        adapm.Config(10, 4, 1, 0, None, None, 0, 3),                 # unknown action timing
+        adapm.Config(10, 4, 1, 0, None, None, 0, 1, 1.5),            # smoothing factor above 1
+        adapm.Config(10, 4, 1, 0, None, None, 0, 1, 0.1, 1.0),       # quantile must be below 1
+        adapm.Config(10, 4, 1, 0, None, None, 0, 1, 0.1, 0.9, -1.0),  # negative initial rate
     ]
     for cfg in bad:
         assert lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h)) == adapm.EINVAL
     assert lib.adapm_intent(None, 0, None, 0, 0, 1) == adapm.EINVAL
     assert lib.adapm_wait(None) == adapm.EINVAL
+
+
+def test_poisson_quantile_of_the_library_equals_the_oracle(lib_path):
+    # the host rule of adaptive action timing (Algorithm 1) against the oracle's, which is pinned to scipy
+    from oracle.timing import poisson_quantile
+    adapm.load(lib_path)
+    for lam in (0.05, 0.7, 1.0, 2.0, 2.8, 9.5, 20.0, 111.1, 2500.0):
+        for p in (0.001, 0.5, 0.9, 0.9999, 1 - 1e-10):
+            assert adapm.poisson_quantile(lam, p) == poisson_quantile(lam, p), (lam, p)
+    with pytest.raises(adapm.AdaPMError):
+        adapm.poisson_quantile(0.0, 0.5)
+    with pytest.raises(adapm.AdaPMError):
+        adapm.poisson_quantile(1.0, 1.0)

@@ -109,14 +109,17 @@ def _mf_small_cfg():
                                batch=700, lookahead=2, zipf_s=1.1, total_cells=10 ** 6)
 
 
-@pytest.mark.parametrize("relocate", [False, True])
-def test_mf_adagrad_zipf(gpu_lib, relocate):
+@pytest.mark.parametrize("relocate,timing", [(False, "start"), (True, "start"), (False, "adaptive"),
+                                             (True, "adaptive")])
+def test_mf_adagrad_zipf(gpu_lib, relocate, timing):
     cfg = _mf_small_cfg()
     nclk = 6
     init = init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
     pm = gpu_lib.ParameterManager(cfg.num_keys, cfg.value_len, cfg.workers,
-                                  init_values=torch.from_numpy(init).cuda(), relocate=relocate)
-    ref = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=relocate)
+                                  init_values=torch.from_numpy(init).cuda(), relocate=relocate,
+                                  action_timing=timing)
+    ref = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=relocate,
+                                 action_timing=timing)
     batches = {(w, c): wl.mf_batch(cfg, w, c) for w in range(cfg.workers)
                for c in range(nclk + cfg.lookahead + 1)}
 
