@@ -24,7 +24,8 @@ the sum invariant with dyadic deltas (bit-exact), hand-worked scenarios in
 tests/golden/, the owner and replica intervals of the paper's Fig. 4b-d and
 Fig. 10a, the owner recomputed by brute force from the call log, the
 Poisson quantile against scipy's, the rate estimate against the closed form
-of its recursion, the
+of its recursion, the versioned refresh equal to the full one in exact
+arithmetic, the
 single-worker reduction to textbook mini-batch SGD,
 fp64 finite-difference gradients, ComplEx scores by complex arithmetic and
 closed forms, Zipf frequencies by chi-square.  No function here is "parity

@@ -37,6 +37,14 @@ Definitions
     acc = 0 (App. B.1.2: the owner merges the updates and propagates them to
     the replica holders; sending only unseen versions gives the same values).
 
+Versioned refresh (App. B.1.2: holders request only the updates they have
+not received).  With delta_refresh=True, sync leaves the value of a replica
+alone when its holder is the key's only holder and nobody else wrote main[k]
+since the last sync that merged k (no write to main without a replica, no
+destroyed replica): the holder has all the updates already, its own.  Its
+pending updates are still merged and cleared.  In exact arithmetic nothing
+changes; in fp32 the holder keeps its own rounding of the same sum.
+
 Action timing (Sec. 4.2).  action_timing="start" (default) acts on an intent
 exactly when it becomes active.  "signal" acts when the intent is signalled
 (the paper's immediate-action ablation, Sec. 5.8): its window is treated as
@@ -83,7 +91,7 @@ def _f32(x):
 
 class ParameterManagerOracle:
     def __init__(self, num_keys, value_len, num_workers, init, relocation=False, action_timing="start",
-                 timing_alpha=None, timing_p=None, timing_lambda0=None):
+                 timing_alpha=None, timing_p=None, timing_lambda0=None, delta_refresh=False):
         init = np.asarray(init, dtype=np.float32)
         if init.shape != (num_keys, value_len):
             raise OracleError("init must have shape (num_keys, value_len)")
@@ -104,6 +112,9 @@ class ParameterManagerOracle:
         kw = {k: v for k, v in (("alpha", timing_alpha), ("p", timing_p), ("lambda0", timing_lambda0))
               if v is not None}
         self.rates = [RateEstimate(**kw) for _ in range(self.W)]
+        self.delta_refresh = bool(delta_refresh)
+        self.changed = np.zeros(self.K, dtype=bool)   # main[k] written other than by a sync merge
+        self.refreshed = 0
 
     # -- argument checks ---------------------------------------------------
     def _check_worker(self, w):
@@ -140,6 +151,7 @@ class ParameterManagerOracle:
     def _destroy(self, w, k):
         val, acc = self.replicas[w].pop(k)
         self.main[k] = _f32(self.main[k].astype(np.float64) + acc.astype(np.float64))
+        self.changed[k] = True
         self.destroyed += 1
 
     def _relocate(self, k, w):
@@ -226,6 +238,7 @@ class ParameterManagerOracle:
                 reps[k] = (_f32(val.astype(np.float64) + s), _f32(acc.astype(np.float64) + s))
             else:
                 self.main[k] = _f32(self.main[k].astype(np.float64) + s)
+                self.changed[k] = True
 
     def sync(self):
         keys = sorted(set().union(*[set(r) for r in self.replicas]))
@@ -235,8 +248,14 @@ class ParameterManagerOracle:
             for w in holders:                        # ascending worker
                 total = total + self.replicas[w][k][1].astype(np.float64)
             self.main[k] = _f32(total)
+            # versioned refresh: a sole holder of a key nobody else wrote since the last sync has
+            # received every update already (its own), so only its pending updates are cleared
+            stale = not self.delta_refresh or len(holders) > 1 or self.changed[k]
             for w in holders:
-                self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+                val = self.main[k].copy() if stale else self.replicas[w][k][0]
+                self.replicas[w][k] = (val, np.zeros(self.D, dtype=np.float32))
+            self.refreshed += len(holders) if stale else 0
+            self.changed[k] = False
         if self.action_timing == "adaptive":
             self._act_in_round()
 
