@@ -49,7 +49,7 @@ METRIC = "pulled+pushed keys/s and training samples/s on 1 GB300; % of HBM roofl
 # the traffic is reported as null.
 PUSH_SOURCES = ("paper_2206_00470_gb300/csrc/push.cu", "paper_2206_00470_gb300/csrc/rowgroup.cuh")
 PUSH_TRAFFIC = {
-    "mf": {"bytes_per_row": 79.213e6 / 65536, "sha256_16": "f902f353c30b86b9"},   # profiles/push_scatter_mf_2Mx200K.md
+    "mf": {"bytes_per_row": 83.35e6 / 65536, "sha256_16": "063dcdafb303627f"},   # profiles/push_scatter_mf_2Mx200K.md
     "micro": {"bytes_per_row": None, "sha256_16": None},
 }
 
@@ -556,8 +556,9 @@ def alg_bytes_per_step(wk, d, steps, relocate=False):
         "push": R * (4 + row) + U * (4 + tgt),
         # the scatter kernel alone also reads the sorted (key, position) pairs
         "push_kernel": R * (8 + row) + U * (4 + tgt),
-        # main += pending (2 rows per key); val := main, pending := 0 (3 rows per replica)
-        "sync": per["sync_keys"] * 2 * row + per["sync_replicas"] * 3 * row,
+        # main += pending (2 rows per key); read pending and clear it (2 rows per replica); val := main
+        # (1 row per refreshed replica: all of them unless the refresh is versioned)
+        "sync": per["sync_keys"] * 2 * row + per["sync_replicas"] * 2 * row + per["sync_refreshed"] * row,
         # destroy: read pending, read+write main; create: read main, write val and pending
         "advance": (per["created"] + per["destroyed"]) * 3 * row,
     }
@@ -572,7 +573,8 @@ def alg_bytes_per_step(wk, d, steps, relocate=False):
     return out
 
 
-COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "created", "destroyed", "relocations")
+COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "sync_refreshed", "created", "destroyed",
+            "relocations")
 
 
 def run_ours(args, ws, rank, local):
@@ -585,7 +587,8 @@ def run_ours(args, ws, rank, local):
     wk.prepare(total_clocks + 2 * args.steps + 2)
     init = wk.init_store()
     pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
-                                relocate=args.relocate, action_timing=args.timing)
+                                relocate=args.relocate, action_timing=args.timing,
+                                delta_refresh=args.delta_refresh)
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -688,6 +691,7 @@ def run_ours(args, ws, rank, local):
         "config": dict(wk.config(), parallelism=f"replicas{ws}",
                        placement="relocate" if args.relocate else "replicate",
                        action_timing=args.timing,
+                       refresh="versioned" if args.delta_refresh else "full",
                        l2="inputs larger than L2 (no flush)"),
         "gpu_launches": int(launches),
         "clocks": clk,
@@ -696,7 +700,7 @@ def run_ours(args, ws, rank, local):
         "stats": {k: stats[k] for k in ("live_replicas", "high_water", "capacity")},
         # replica management per step (profiled pass): what relocation saves against always replicating
         "replica_events_per_step": {k: delta[k] / steps for k in ("created", "destroyed", "sync_replicas",
-                                                                   "sync_keys", "relocations")},
+                                                                   "sync_refreshed", "sync_keys", "relocations")},
         "setup_s": setup_s,
     }
     if e2e_ms is not None:
@@ -729,7 +733,7 @@ def oracle_sample(workload, budget_s, args):
         rel = {k: np.searchsorted(touched, v) for k, v in kmap.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.value_len, cfg.seed, cfg.init_std)
         pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
-                                    action_timing=args.timing)
+                                    action_timing=args.timing, delta_refresh=args.delta_refresh)
         g = np.random.default_rng(0)
         deltas = (g.standard_normal((cfg.batch, cfg.value_len)) * cfg.delta_std).astype(np.float32)
 
@@ -763,7 +767,7 @@ def oracle_sample(workload, budget_s, args):
                for k, (a, b, v) in data.items()}
         init = hashgen.init_rows_np(touched, cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
         pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
-                                    action_timing=args.timing)
+                                    action_timing=args.timing, delta_refresh=args.delta_refresh)
 
         def work(w, cl):
             a, b, v = rel[(w, cl)]
@@ -787,7 +791,7 @@ def oracle_sample(workload, budget_s, args):
         nclk = wl.tiny_mf_clocks(cfg, data[3])
         init = hashgen.init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
         pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, cfg.workers, init, relocation=args.relocate,
-                                    action_timing=args.timing)
+                                    action_timing=args.timing, delta_refresh=args.delta_refresh)
         bt = {(w, c): [x.numpy() for x in wl.tiny_mf_batch(cfg, data, w, c)]
               for w in range(cfg.workers) for c in range(nclk + cfg.lookahead + 1)}
 
@@ -827,7 +831,7 @@ def oracle_sample(workload, budget_s, args):
         theta = cfg.theta_dim if workload == "complex" else cfg.dim
         init = hashgen.init_rows_np(touched, cfg.value_len, theta, cfg.seed, cfg.init_std)
         pm = ParameterManagerOracle(touched.size, cfg.value_len, cfg.workers, init, relocation=args.relocate,
-                                    action_timing=args.timing)
+                                    action_timing=args.timing, delta_refresh=args.delta_refresh)
         rel = lambda x: np.searchsorted(touched, x)  # noqa: E731
 
         if workload == "complex":
@@ -913,6 +917,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--relocate", action="store_true",
                     help="relocate a key to its only worker with active intent instead of always replicating")
+    ap.add_argument("--delta-refresh", action="store_true",
+                    help="versioned refresh: sync leaves a sole holder's value when nobody else wrote the key")
     ap.add_argument("--timing", default="start", choices=["start", "adaptive", "signal"],
                     help="act on an intent at its start clock, by Algorithm 1 at each sync, or when signalled")
     args = ap.parse_args()

@@ -5,11 +5,12 @@
  * Signaling" (arXiv 2206.00470).  Workers announce, through Intent(), which
  * keys they will access in a window of their own logical clock (Sec. 3).  The
  * manager keeps a replica of each such key at the worker for exactly the
- * span of the intent (Sec. 4.1, selective replication; this library always
- * replicates, the paper's "AdaPM w/o relocation" of Sec. 5.5), serves the
- * worker's reads from the replica, accumulates the worker's writes in it, and
- * merges the accumulated updates into the main copy when the replica is
- * destroyed or when sync() runs (App. B.1.2).  Access without intent is
+ * span of the intent (Sec. 4.1, selective replication; by default for every
+ * active intent, the paper's "AdaPM w/o relocation" of Sec. 5.5, or with
+ * relocation when one worker alone has active intent, see adapm_create),
+ * serves the worker's reads from the replica, accumulates the worker's writes
+ * in it, and merges the accumulated updates into the main copy when the
+ * replica is destroyed or when sync() runs (App. B.1.2).  Access without intent is
  * allowed at any time and goes to the main copy (Sec. 4, "optional intent").
  * W workers are worker slots that share one GPU.
  *
@@ -18,7 +19,9 @@
  *     row-major, value_len a multiple of 4 (16-byte rows).
  *   - Array arguments may be device pointers or host pointers (pinned or
  *     pageable); the library detects which with cudaPointerGetAttributes.
- *     Host inputs are copied to the device on the library stream; a host
+ *     Host inputs are copied to the device before the call's kernels (pinned
+ *     ones on a copy stream of the library's, so that the copy overlaps the
+ *     kernels of earlier calls; the library stream waits for it); a host
  *     output is filled by a device-to-host copy on the library stream.
  *   - Calls are ordered on the library stream and return once their work is
  *     enqueued.  Device and pinned host arrays are read and written in
@@ -79,6 +82,8 @@ typedef struct {
   double timing_alpha;       /* ADAPM_ACT_ADAPTIVE: smoothing factor, 0 = 0.1 */
   double timing_p;           /* ADAPM_ACT_ADAPTIVE: Poisson quantile, 0 = 0.9999 */
   double timing_lambda0;     /* ADAPM_ACT_ADAPTIVE: initial clocks per round, 0 = 10 */
+  int32_t delta_refresh;     /* 0: sync refreshes every replica; 1: versioned refresh (see
+                                adapm_sync) */
 } adapm_config;
 
 /* Action timing (Sec. 4.2).
@@ -104,7 +109,8 @@ typedef struct {
 /* Create a manager: main store = init_values, every clock 0, no intents, no
  * replicas, every key at its home (owned by no worker).  Memory: K*D*4 (main)
  * + W*K*8 (slot maps, refcounts) + K*8 (holder masks, intent stamps) + K*2
- * with relocate (owner and active-worker count) + capacity*(2*D*4 + 12)
+ * with relocate (owner and active-worker count) + K with delta_refresh
+ * (written-since-sync flags) + capacity*(2*D*4 + 12)
  * bytes of device memory.  Returns ADAPM_ENOMEM if it does not fit.
  *
  * Relocation (relocate = 1).  Every key has an owner: its home at first,
@@ -182,8 +188,15 @@ adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, const uint32_t*
 /* Replica synchronisation (App. B.1.2): for every key with replicas,
  * main += the pending updates of all holders (ascending worker order), then
  * every holder's replica := main and its pending updates := 0.  With
- * ADAPM_ACT_ADAPTIVE this is also a communication round of Algorithm 1
- * (see adapm_config), which may activate intents early. */
+ * delta_refresh = 1 (App. B.1.2: holders receive only the updates they have
+ * not seen) the value of a key's only replica is left as it is when nobody
+ * else wrote the key since its last sync (no write to main by a worker
+ * without a replica, no destroyed replica): that holder has every update
+ * already, its own, so only its pending updates are merged and cleared.
+ * Exact arithmetic gives the same values; in fp32 the holder keeps its own
+ * rounding of the same sum.  With ADAPM_ACT_ADAPTIVE a sync is also a
+ * communication round of Algorithm 1 (see adapm_config), which may activate
+ * intents early. */
 adapm_status adapm_sync(adapm_ctx* ctx);
 
 /* Block until the stream is idle; return and clear the first sticky device
@@ -266,6 +279,7 @@ typedef struct {
   uint64_t sync_keys;        /* keys merged by sync, cumulative */
   uint64_t sync_replicas;    /* replicas refreshed by sync, cumulative */
   uint64_t relocations;      /* owner changes, cumulative (relocation only) */
+  uint64_t sync_refreshed;   /* replica values written by sync, cumulative */
 } adapm_stats;
 
 adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);

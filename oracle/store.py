@@ -40,8 +40,9 @@ Definitions
 Versioned refresh (App. B.1.2: holders request only the updates they have
 not received).  With delta_refresh=True, sync leaves the value of a replica
 alone when its holder is the key's only holder and nobody else wrote main[k]
-since the last sync that merged k (no write to main without a replica, no
-destroyed replica): the holder has all the updates already, its own.  Its
+since the last sync that merged k or the last replica creation of k (no
+write to main without a replica, no destroyed replica): the holder has all
+the updates already, its own.  Its
 pending updates are still merged and cleared.  In exact arithmetic nothing
 changes; in fp32 the holder keeps its own rounding of the same sum.
 
@@ -146,6 +147,10 @@ class ParameterManagerOracle:
 
     def _create(self, w, k):
         self.replicas[w][k] = (self.main[k].copy(), np.zeros(self.D, dtype=np.float32))
+        # a new replica has seen every update; a replica of another worker that has not is refreshed at
+        # the next sync anyway, since the key then has several holders, or becomes the only one by the
+        # destruction of this one, which marks the key again
+        self.changed[k] = False
         self.created += 1
 
     def _destroy(self, w, k):

@@ -44,6 +44,7 @@ class Config(ctypes.Structure):
         ("timing_alpha", ctypes.c_double),
         ("timing_p", ctypes.c_double),
         ("timing_lambda0", ctypes.c_double),
+        ("delta_refresh", ctypes.c_int32),
     ]
 
 
@@ -63,6 +64,7 @@ class Stats(ctypes.Structure):
         ("sync_keys", ctypes.c_uint64),
         ("sync_replicas", ctypes.c_uint64),
         ("relocations", ctypes.c_uint64),
+        ("sync_refreshed", ctypes.c_uint64),
     ]
 
 
@@ -193,7 +195,7 @@ class ParameterManager:
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
                  stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
-                 timing_lambda0=0.0):
+                 timing_lambda0=0.0, delta_refresh=False):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -212,7 +214,7 @@ class ParameterManager:
         self.action_timing = action_timing
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
                      ctypes.c_void_p(handle), int(self.relocate), ACTION_TIMING[action_timing],
-                     float(timing_alpha), float(timing_p), float(timing_lambda0))
+                     float(timing_alpha), float(timing_p), float(timing_lambda0), int(bool(delta_refresh)))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:

@@ -297,6 +297,7 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s
         if (col < D4) atomicAdd(main4 + (uint64_t)k * D4 + col, ac[r][c]);
       }
       if (lane == 0) {
+        if (s.dirty != nullptr) s.dirty[k] = 1;   // versioned refresh: main changed
         s.map[(uint64_t)a * s.K + k] = -1;
         atomicAnd(s.holders + k, ~(1u << a));
         s.slot_owner[sl[r]] = kEmptySlot;
@@ -386,6 +387,9 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store 
         }
       }
       if (lane == 0) {
+        // versioned refresh: the new replica has seen every update (a stale
+        // replica of another worker is refreshed anyway: the key has two holders)
+        if (s.dirty != nullptr) s.dirty[k[r]] = 0;
         mapw[k[r]] = sl[r];
         atomicOr(s.holders + k[r], 1u << w);
         s.slot_owner[sl[r]] = ((unsigned long long)w << 32) | k[r];

@@ -11,6 +11,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <deque>
 #include <map>
 #include <new>
 #include <string>
@@ -70,6 +71,20 @@ struct adapm_ctx {
   std::vector<cudaEvent_t> spare_events;
   double prof_ms[ADAPM_NUM_OPS] = {0};
   uint64_t prof_calls[ADAPM_NUM_OPS] = {0};
+  // Pinned host inputs are copied on a stream of their own from a pool of
+  // their own, so that a call's copies overlap the kernels of the calls
+  // enqueued before it.  `stream` waits for each copy (event `staged`).  A
+  // mark (an event on `stream` with the bytes staged before it) is taken at
+  // each staging call; while more than kStageAhead bytes are staged beyond
+  // the oldest mark, copy_in waits for that mark, which bounds the staging
+  // memory in flight.
+  cudaStream_t copy_in = nullptr;
+  cudaMemPool_t stage_pool = nullptr;
+  cudaEvent_t staged = nullptr;
+  std::deque<std::pair<cudaEvent_t, uint64_t>> stage_marks;
+  std::vector<cudaEvent_t> spare_marks;
+  uint64_t stage_unmarked = 0;   // bytes staged since the last mark
+  uint64_t stage_live = 0;       // bytes staged since the oldest mark
 };
 
 namespace {
@@ -97,13 +112,79 @@ adapm_status cuda_fail(adapm_ctx* c, cudaError_t e, const char* where) {
     if (e_ != cudaSuccess) return cuda_fail(ctx, e_, #call); \
   } while (0)
 
-bool is_device_ptr(const void* p) {
+enum class MemKind { Device, PinnedHost, PageableHost };
+
+MemKind mem_kind(const void* p) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
     cudaGetLastError();
-    return false;
+    return MemKind::PageableHost;
   }
-  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return MemKind::Device;
+  return a.type == cudaMemoryTypeHost ? MemKind::PinnedHost : MemKind::PageableHost;
+}
+
+bool is_device_ptr(const void* p) { return mem_kind(p) == MemKind::Device; }
+
+constexpr uint64_t kStageAhead = 8ull << 30;   // staged input bytes ahead of the kernels, at most
+
+// The staging stream and pool, made on the first pinned host input: their own
+// stream, and a pool that reuses a block only once its free is known to be
+// done, never by making copy_in wait for `stream` on its own.
+cudaError_t ensure_copy_in(adapm_ctx* ctx) {
+  if (ctx->copy_in) return cudaSuccess;
+  cudaMemPoolProps props{};
+  props.allocType = cudaMemAllocationTypePinned;
+  props.location.type = cudaMemLocationTypeDevice;
+  props.location.id = ctx->device;
+  cudaError_t e = cudaMemPoolCreate(&ctx->stage_pool, &props);
+  if (e != cudaSuccess) return e;
+  uint64_t keep = ~0ull;
+  int no = 0;
+  if ((e = cudaMemPoolSetAttribute(ctx->stage_pool, cudaMemPoolAttrReleaseThreshold, &keep)) != cudaSuccess ||
+      (e = cudaMemPoolSetAttribute(ctx->stage_pool, cudaMemPoolReuseAllowInternalDependencies, &no)) !=
+          cudaSuccess ||
+      (e = cudaEventCreateWithFlags(&ctx->staged, cudaEventDisableTiming)) != cudaSuccess)
+    return e;
+  return cudaStreamCreateWithFlags(&ctx->copy_in, cudaStreamNonBlocking);
+}
+
+// Take a mark on `stream` for the bytes staged since the last one, then let
+// copy_in wait for the oldest marks while too much is staged beyond them.
+cudaError_t stage_mark(adapm_ctx* ctx, uint64_t next_bytes) {
+  cudaError_t e = cudaSuccess;
+  // marks already passed release their bytes without a wait
+  while (!ctx->stage_marks.empty()) {
+    const cudaError_t q = cudaEventQuery(ctx->stage_marks.front().first);
+    if (q == cudaErrorNotReady) {
+      if (cudaPeekAtLastError() == cudaErrorNotReady) cudaGetLastError();
+      break;
+    }
+    if (q != cudaSuccess) return q;
+    ctx->spare_marks.push_back(ctx->stage_marks.front().first);
+    ctx->stage_live -= ctx->stage_marks.front().second;
+    ctx->stage_marks.pop_front();
+  }
+  if (ctx->stage_unmarked) {
+    cudaEvent_t ev = nullptr;
+    if (!ctx->spare_marks.empty()) {
+      ev = ctx->spare_marks.back();
+      ctx->spare_marks.pop_back();
+    } else if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess) {
+      return e;
+    }
+    if ((e = cudaEventRecord(ev, ctx->stream)) != cudaSuccess) return e;
+    ctx->stage_marks.emplace_back(ev, ctx->stage_unmarked);
+    ctx->stage_unmarked = 0;
+  }
+  while (!ctx->stage_marks.empty() && ctx->stage_live + next_bytes > kStageAhead) {
+    auto m = ctx->stage_marks.front();
+    ctx->stage_marks.pop_front();
+    if ((e = cudaStreamWaitEvent(ctx->copy_in, m.first, 0)) != cudaSuccess) return e;
+    ctx->spare_marks.push_back(m.first);   // the wait has captured it; it can be recorded again
+    ctx->stage_live -= m.second;
+  }
+  return cudaSuccess;
 }
 
 template <class T>
@@ -130,14 +211,30 @@ cudaError_t stage_in(adapm_ctx* ctx, const T* p, size_t count, Input<T>* in) {
     in->dev = p;
     return cudaSuccess;
   }
-  if (is_device_ptr(p)) {
+  const MemKind kind = mem_kind(p);
+  if (kind == MemKind::Device) {
     in->dev = p;
     return cudaSuccess;
+  }
+  const uint64_t bytes = count * sizeof(T);
+  if (kind == MemKind::PinnedHost) {
+    cudaError_t e = ensure_copy_in(ctx);
+    if (e == cudaSuccess) e = stage_mark(ctx, bytes);
+    if (e != cudaSuccess) return e;
+    e = cudaMallocFromPoolAsync(reinterpret_cast<void**>(&in->owned), bytes, ctx->stage_pool, ctx->copy_in);
+    if (e != cudaSuccess) return e;
+    in->dev = in->owned;
+    e = cudaMemcpyAsync(in->owned, p, bytes, cudaMemcpyHostToDevice, ctx->copy_in);
+    if (e == cudaSuccess) e = cudaEventRecord(ctx->staged, ctx->copy_in);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(ctx->stream, ctx->staged, 0);
+    ctx->stage_unmarked += bytes;
+    ctx->stage_live += bytes;
+    return e;   // the buffer is freed on `stream` after its consumer, like any pool buffer
   }
   cudaError_t e = pool_alloc(ctx, &in->owned, count);
   if (e != cudaSuccess) return e;
   in->dev = in->owned;
-  return cudaMemcpyAsync(in->owned, p, count * sizeof(T), cudaMemcpyHostToDevice, ctx->stream);
+  return cudaMemcpyAsync(in->owned, p, bytes, cudaMemcpyHostToDevice, ctx->stream);
 }
 
 // Device buffer for an output array; copied out to host arrays at finish.
@@ -348,7 +445,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       cfg->num_workers > (uint32_t)kMaxWorkers || (cfg->relocate != 0 && cfg->relocate != 1) ||
       cfg->action_timing < ADAPM_ACT_AT_START || cfg->action_timing > ADAPM_ACT_ON_SIGNAL ||
       !(cfg->timing_alpha >= 0.0 && cfg->timing_alpha <= 1.0) ||
-      !(cfg->timing_p >= 0.0 && cfg->timing_p < 1.0) || !(cfg->timing_lambda0 >= 0.0))
+      !(cfg->timing_p >= 0.0 && cfg->timing_p < 1.0) || !(cfg->timing_lambda0 >= 0.0) ||
+      (cfg->delta_refresh != 0 && cfg->delta_refresh != 1))
     return ADAPM_EINVAL;
   adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
   if (!ctx) return ADAPM_ENOMEM;
@@ -380,6 +478,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   if (cudaMemPoolCreate(&ctx->pool, &props) != cudaSuccess) return bail(ADAPM_ECUDA);
   uint64_t keep = ~0ull;
   cudaMemPoolSetAttribute(ctx->pool, cudaMemPoolAttrReleaseThreshold, &keep);
+
   ctx->bits = bits_for(K);
   Store& s = ctx->s;
   s.K = K;
@@ -392,6 +491,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       !dmalloc((void**)&s.rc, W * K * 4) || !dmalloc((void**)&s.holders, K * 4) ||
       !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
       !dmalloc((void**)&s.stamp, K * 4) || (cfg->relocate && !dmalloc((void**)&s.own, K * 2)) ||
+      (cfg->delta_refresh && !dmalloc((void**)&s.dirty, K)) ||
       !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
     cudaGetLastError();
     return bail(ADAPM_ENOMEM);
@@ -409,6 +509,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   ok &= cudaMemsetAsync(s.holders, 0, K * 4, st) == cudaSuccess;
   ok &= cudaMemsetAsync(s.stamp, 0, K * 4, st) == cudaSuccess;   // intent tags start at 1
   if (s.own) ok &= cudaMemsetAsync(s.own, 0, K * 2, st) == cudaSuccess;   // home, no active worker
+  if (s.dirty) ok &= cudaMemsetAsync(s.dirty, 0, K, st) == cudaSuccess;
   DevState h{};
   h.free_top = (int32_t)S;
   ok &= cudaMemcpyAsync(ctx->dstate, &h, sizeof h, cudaMemcpyHostToDevice, st) == cudaSuccess;
@@ -428,7 +529,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
-                  s.stamp, s.own, ctx->dstate};
+                  s.stamp, s.own, s.dirty, ctx->dstate};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& t : ctx->pending) {
@@ -436,6 +537,12 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
     cudaEventDestroy(std::get<2>(t));
   }
   for (auto e : ctx->spare_events) cudaEventDestroy(e);
+  if (ctx->copy_in) cudaStreamSynchronize(ctx->copy_in);
+  for (auto& m : ctx->stage_marks) cudaEventDestroy(m.first);
+  for (auto e : ctx->spare_marks) cudaEventDestroy(e);
+  if (ctx->staged) cudaEventDestroy(ctx->staged);
+  if (ctx->copy_in) cudaStreamDestroy(ctx->copy_in);
+  if (ctx->stage_pool) cudaMemPoolDestroy(ctx->stage_pool);
   if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
   if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
   cudaGetLastError();
@@ -885,6 +992,7 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
   out->sync_keys = h.sync_keys;
   out->sync_replicas = h.sync_replicas;
   out->relocations = h.relocations;
+  out->sync_refreshed = h.sync_refreshed;
   return ADAPM_OK;
 }
 

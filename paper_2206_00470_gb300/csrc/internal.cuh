@@ -9,6 +9,8 @@
 //   slot_owner  [S]    uint64   (w << 32) | k of a live slot, kEmptySlot if free
 //   free_stack  [S]    int32    free slots, top at free_stack[free_top - 1]
 //   stamp       [K]    uint32   tag of the last Intent call that listed k
+//   dirty       [K]    uint8    versioned refresh only: main[k] written other
+//                               than by a sync merge since the last sync of k
 //   own         [K]    uint16   relocation mode only: ((owner + 1) << 8) |
 //                               number of workers with active intent; owner
 //                               -1 is the key's home (no worker held it yet)
@@ -52,6 +54,7 @@ struct DevState {
   unsigned long long sync_keys;       // keys merged by sync (cumulative)
   unsigned long long sync_replicas;   // replicas refreshed by sync (cumulative)
   unsigned long long relocations;     // owner changes (relocation mode, cumulative)
+  unsigned long long sync_refreshed;  // replica values written by sync (cumulative)
   // grid barriers of the sort: blocks arrived, over the context's lifetime
   // (a line of its own, away from the counters above)
   alignas(128) unsigned long long bar_arrivals;
@@ -68,7 +71,8 @@ struct Store {
   unsigned long long* slot_owner;
   int32_t* free_stack;
   uint32_t* stamp;
-  uint16_t* own;   // null unless relocation mode
+  uint16_t* own;    // null unless relocation mode
+  uint8_t* dirty;   // null unless versioned refresh
   DevState* st;
   uint64_t K;
   uint64_t S;

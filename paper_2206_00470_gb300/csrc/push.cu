@@ -40,6 +40,8 @@ __device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, u
       const uint32_t col = lane + c * G;
       if (col < D4) atomicAdd(t2 + col, sum[c]);
     }
+  } else if (s.dirty != nullptr && lane == 0) {
+    s.dirty[k] = 1;   // versioned refresh: main written by a worker without a replica
   }
 }
 
@@ -107,7 +109,11 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
         f = (piece_end ? 1 : 0) | (started ? 2 : 0) | (seg_end ? 4 : 0) |
             ((seg_begin || i == cs) ? 8 : 0) | 16;
         if (seg_begin) ++heads;
-        if ((f & 7) == 7) slot = mapw[k];
+        if ((f & 7) == 7) {
+          slot = mapw[k];
+          // versioned refresh: main written by a worker without a replica
+          if (slot < 0 && s.dirty != nullptr) s.dirty[k] = 1;
+        }
       }
       sf[i] = f;
       ss[i] = slot;

@@ -87,8 +87,9 @@ pull_kernel(Store s, int w, const uint32_t* __restrict__ keys, uint64_t n, float
 // ---------------------------------------------------------------------------
 // sync
 // ---------------------------------------------------------------------------
-template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s) {
+// VER: versioned refresh (s.dirty is set)
+template <int G, int C, bool VER>
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : (VER && C == 1 ? 3 : 4)) sync_kernel(Store s) {
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
   const uint64_t hw = (uint64_t)s.st->high_water;
@@ -96,10 +97,13 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
-  uint32_t nkeys = 0, nreps = 0;
+  uint32_t nkeys = 0, nreps = 0, nref = 0;   // nref: VER only
   // R slots per group at a time: owners, holder masks, then (for keys held
   // by one worker only, the common case) main and pending rows, each as one
-  // round of independent loads
+  // round of independent loads.  Versioned refresh (App. B.1.2: a holder
+  // receives only updates it has not seen): a sole holder's value is left
+  // alone unless main[k] was written other than by a sync since the last
+  // sync of k (dirty[k]); keys with several holders are always refreshed.
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
   for (uint64_t b = g * R; b < hw; b += ng * R) {
     unsigned long long own[R];
@@ -108,35 +112,42 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
     for (int r = 0; r < R; ++r) own[r] = b + r < hw ? s.slot_owner[b + r] : kEmptySlot;
 #pragma unroll
     for (int r = 0; r < R; ++r) mk[r] = own[r] != kEmptySlot ? s.holders[(uint32_t)own[r]] : 0u;
-    bool single[R];
+    // a live slot's key is held by this worker alone iff its mask has one bit
+    // (its own); such a mask is known, so it is replaced by the refresh flag
+    // (1: write the value, 0: leave it), which keeps at most one bit set
+    auto is_single = [&](int r) { return own[r] != kEmptySlot && __popc(mk[r]) <= 1; };
     float4 mv[R][C], av[R][C];
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      const uint32_t w = (uint32_t)(own[r] >> 32);
-      single[r] = own[r] != kEmptySlot && mk[r] == (1u << w);
+      const bool single = is_single(r);
+      if (VER && single) mk[r] = (uint32_t)s.dirty[(uint32_t)own[r]];
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        const bool cv = single[r] && col < D4;
+        const bool cv = single && col < D4;
         mv[r][c] = cv ? main4[(uint64_t)(uint32_t)own[r] * D4 + col] : f4zero();
         av[r][c] = cv ? acc4[(b + r) * D4 + col] : f4zero();
       }
     }
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      if (!single[r]) continue;
+      if (!is_single(r)) continue;
+      const uint32_t k = (uint32_t)own[r];
       if (lane == 0) {
         nkeys += 1;
         nreps += 1;
+        if (VER && mk[r]) {
+          nref += 1;
+          s.dirty[k] = 0;
+        }
       }
-      const uint32_t k = (uint32_t)own[r];
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
         if (col < D4) {
           const float4 m = f4add(mv[r][c], av[r][c]);
           main4[(uint64_t)k * D4 + col] = m;
-          val4[(b + r) * D4 + col] = m;
+          if (!VER || mk[r]) val4[(b + r) * D4 + col] = m;
           acc4[(b + r) * D4 + col] = f4zero();
         }
       }
@@ -144,7 +155,7 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
     // keys with several holders: the lowest holder merges all of them
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      if (own[r] == kEmptySlot || single[r]) continue;
+      if (own[r] == kEmptySlot || is_single(r)) continue;
       const uint32_t w = (uint32_t)(own[r] >> 32);
       const uint32_t k = (uint32_t)own[r];
       const uint32_t mask = mk[r];
@@ -152,6 +163,10 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
       if (lane == 0) {
         nkeys += 1;
         nreps += (uint32_t)__popc(mask);
+        if (VER) {
+          nref += (uint32_t)__popc(mask);
+          s.dirty[k] = 0;
+        }
       }
       float4 m[C];
 #pragma unroll
@@ -209,9 +224,15 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) sync_kernel(Store s)
     }
   }
   block_sum2(nkeys, nreps);
+  if (VER) {
+    __syncthreads();   // block_sum2's shared words are reused below
+    uint32_t unused = 0;
+    block_sum2(nref, unused);
+  }
   if (threadIdx.x == 0 && nkeys) {
     atomicAdd(&s.st->sync_keys, (unsigned long long)nkeys);
     atomicAdd(&s.st->sync_replicas, (unsigned long long)nreps);
+    atomicAdd(&s.st->sync_refreshed, (unsigned long long)(VER ? nref : nreps));
   }
 }
 
@@ -292,7 +313,11 @@ void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stre
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     note_launches(1);
     constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // slots per group, as in sync_kernel
-    sync_kernel<G, C><<<grid_for((slot_bound + R - 1) / R, G, sms), kThreads, 0, stream>>>(s);
+    const unsigned grid = grid_for((slot_bound + R - 1) / R, G, sms);
+    if (s.dirty != nullptr)
+      sync_kernel<G, C, true><<<grid, kThreads, 0, stream>>>(s);
+    else
+      sync_kernel<G, C, false><<<grid, kThreads, 0, stream>>>(s);
   });
 }
 

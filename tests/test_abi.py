@@ -66,6 +66,7 @@ def test_create_rejects_bad_configs_without_touching_the_gpu(lib_path):
         adapm.Config(10, 4, 1, 0, None, None, 0, 1, 1.5),            # smoothing factor above 1
         adapm.Config(10, 4, 1, 0, None, None, 0, 1, 0.1, 1.0),       # quantile must be below 1
         adapm.Config(10, 4, 1, 0, None, None, 0, 1, 0.1, 0.9, -1.0),  # negative initial rate
+        adapm.Config(10, 4, 1, 0, None, None, 0, 0, 0.0, 0.0, 0.0, 5),  # delta_refresh is 0 or 1
     ]
     for cfg in bad:
         assert lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h)) == adapm.EINVAL

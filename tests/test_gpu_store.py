@@ -246,6 +246,38 @@ def test_host_and_device_arguments_agree(gpu_lib):
         assert np.array_equal(r[0], results[0][0]) and np.array_equal(r[1], results[0][1])
 
 
+def test_pinned_inputs_copied_ahead_of_the_kernels(gpu_lib):
+    # pinned host inputs are copied on a stream of their own that runs ahead of the kernels: a long
+    # sequence enqueued without waits must give exactly the state of the same calls with device arrays
+    K, D, W = 20000, 16, 4
+    init = dyadic_init(K, D, 12)
+    rng = np.random.default_rng(12)
+    calls = []
+    for c in range(30):
+        for w in range(W):
+            k = rng.integers(0, K, size=3000)
+            calls.append((w, c, k, (rng.integers(-64, 65, size=(3000, D)) * 2.0 ** -10).astype(np.float32)))
+    states = []
+    for pinned in (False, True):
+        pm = gpu_lib.ParameterManager(K, D, W, init_values=torch.from_numpy(init).cuda())
+        conv = ((lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()) if pinned
+                else (lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()))
+        args = [(w, c, conv(k.astype(np.int32)), conv(d)) for w, c, k, d in calls]   # kept alive until wait
+        outs = []
+        for w, c, kk, dd in args:
+            pm.intent(w, kk, c + 1, c + 2)
+            outs.append(pm.pull(w, kk))
+            pm.push(w, kk, dd)
+            pm.advance_clock(w)
+            if w == W - 1:
+                pm.sync()
+        pm.wait()
+        states.append(([o.cpu().numpy() for o in outs], pm.read_main(np.arange(K))))
+        pm.close()
+    assert all(np.array_equal(a, b) for a, b in zip(states[0][0], states[1][0]))
+    assert np.array_equal(states[0][1], states[1][1])
+
+
 def test_errors_and_degenerate_inputs(gpu_lib):
     A = gpu_lib
     K, D, W = 50, 8, 2
