@@ -577,6 +577,12 @@ COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "sync_refr
             "relocations")
 
 
+def manager_options(args):
+    """The parameter manager's placement, action timing and refresh options, as named in `config`."""
+    return {"placement": "relocate" if args.relocate else "replicate", "action_timing": args.timing,
+            "refresh": "versioned" if args.delta_refresh else "full"}
+
+
 def run_ours(args, ws, rank, local):
     from paper_2206_00470_gb300 import adapm
     device = torch.device("cuda", local)
@@ -688,10 +694,7 @@ def run_ours(args, ws, rank, local):
         "warmup": args.warmup, "ms_per_step": ms_max / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "samples_per_s": samples if wk.samples_per_step else None,
-        "config": dict(wk.config(), parallelism=f"replicas{ws}",
-                       placement="relocate" if args.relocate else "replicate",
-                       action_timing=args.timing,
-                       refresh="versioned" if args.delta_refresh else "full",
+        "config": dict(wk.config(), parallelism=f"replicas{ws}", **manager_options(args),
                        l2="inputs larger than L2 (no flush)"),
         "gpu_launches": int(launches),
         "clocks": clk,
@@ -884,15 +887,12 @@ def run_reference(args, ws, rank):
     if rank != 0:
         return None
     base = cpu_baseline(args)
-    t_steps = []
-    for _ in range(args.steps):
-        t_steps.append(base["value"])
     line = {
         "impl": "reference", "metric": METRIC, "value": base["value"], "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": dict(WORKLOADS[args.workload](args, None).config(), parallelism="replicas1",
-                       reference="CPU oracle (plain Python/numpy, 1 core)"),
+                       **manager_options(args), reference="CPU oracle (plain Python/numpy, 1 core)"),
         "cpu_baseline": base,
         "e2e": {"value": base["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }

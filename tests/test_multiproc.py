@@ -60,3 +60,16 @@ def test_reference_arm_under_torchrun_prints_once():
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle"
     assert d["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_reference_arm_with_relocation_timing_and_versioned_refresh():
+    # the placement, timing and refresh options reach the oracle the reference arm times
+    cmd = [sys.executable, "bench.py", "--impl", "reference", "--workload", "tiny_mf", "--steps", "3",
+           "--warmup", "3", "--cpu-budget", "1", "--relocate", "--timing", "adaptive", "--delta-refresh"]
+    env = dict(os.environ, OMP_NUM_THREADS="1")
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    d = json.loads([ln for ln in r.stdout.splitlines() if ln.startswith("{")][0])
+    assert d["impl"] == "reference" and d["value"] > 0
+    assert (d["config"]["placement"], d["config"]["action_timing"], d["config"]["refresh"]) == (
+        "relocate", "adaptive", "versioned")
