@@ -139,7 +139,8 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
   constexpr int Q = 4;
   __shared__ uint32_t base_s;
   uint32_t* rcw = s.rc + (uint64_t)w * s.K;
-  const int32_t* mapw = s.map + (uint64_t)w * s.K;
+  int32_t* mapw_mut = s.map + (uint64_t)w * s.K;
+  const int32_t* mapw = mapw_mut;
   uint32_t* counter = START ? &s.st->n_create : &s.st->n_evict;
   const bool reloc = s.own != nullptr;
   uint32_t pre[kEventLists + 1];
@@ -226,6 +227,10 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
         // a key whose replica was never created (capacity exhausted) has nothing to destroy
         hit[q] = sl[q] >= 0;
         e0[q] = (uint32_t)sl[q];
+        // always replicating, the slot map entry is cleared here, where its line was just read
+        // (nothing reads the map between this kernel and the eviction of the listed slot); with
+        // relocation the eviction clears it, off this kernel's longer chain of dependent accesses
+        if (hit[q] && !reloc) mapw_mut[k[q]] = -1;
       }
     }
     uint32_t c = 0, total, mtotal;
@@ -298,7 +303,8 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s
       }
       if (lane == 0) {
         if (s.dirty != nullptr) s.dirty[k] = 1;   // versioned refresh: main changed
-        s.map[(uint64_t)a * s.K + k] = -1;
+        // (always replicating, the events kernel that listed the slot has cleared its map entry)
+        if (s.own != nullptr) s.map[(uint64_t)a * s.K + k] = -1;
         atomicAnd(s.holders + k, ~(1u << a));
         s.slot_owner[sl[r]] = kEmptySlot;
         s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
