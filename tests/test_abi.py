@@ -24,7 +24,7 @@ def lib_path():
     return libbuild.build()
 
 
-def test_header_declares_the_north_star_calls():
+def test_header_declares_the_method_calls():
     names = declared_functions()
     for n in ("adapm_create", "adapm_intent", "adapm_advance_clock", "adapm_pull", "adapm_push",
               "adapm_sync"):
