@@ -85,3 +85,31 @@ def test_poisson_quantile_of_the_library_equals_the_oracle(lib_path):
         adapm.poisson_quantile(0.0, 0.5)
     with pytest.raises(adapm.AdaPMError):
         adapm.poisson_quantile(1.0, 1.0)
+
+
+def test_header_is_plain_c(tmp_path):
+    # the boundary is a C ABI: the header must compile as C (no C++ constructs) and link against the library
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    src = tmp_path / "use_adapm.c"
+    src.write_text(
+        '#include "adapm.h"\n'
+        "int main(void) {\n"
+        "  adapm_config cfg = {0};\n"
+        "  adapm_ctx* ctx = 0;\n"
+        "  int64_t q = 0;\n"
+        "  cfg.num_keys = 0;  /* invalid: rejected before any GPU work */\n"
+        "  if (adapm_create(&cfg, &ctx) != ADAPM_EINVAL) return 1;\n"
+        "  if (adapm_poisson_quantile(20.0, 0.9999, &q) != ADAPM_OK || q != 39) return 2;\n"
+        "  return 0;\n"
+        "}\n")
+    lib = libbuild.build()
+    exe = tmp_path / "use_adapm"
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe),
+                        lib, "-Wl,-rpath," + os.path.dirname(lib)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0, (r.returncode, r.stderr)
