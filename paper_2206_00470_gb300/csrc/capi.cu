@@ -137,16 +137,26 @@ cudaError_t ensure_copy_in(adapm_ctx* ctx) {
   props.allocType = cudaMemAllocationTypePinned;
   props.location.type = cudaMemLocationTypeDevice;
   props.location.id = ctx->device;
-  cudaError_t e = cudaMemPoolCreate(&ctx->stage_pool, &props);
-  if (e != cudaSuccess) return e;
+  cudaMemPool_t pool = nullptr;
+  cudaEvent_t ev = nullptr;
+  cudaStream_t st = nullptr;
   uint64_t keep = ~0ull;
   int no = 0;
-  if ((e = cudaMemPoolSetAttribute(ctx->stage_pool, cudaMemPoolAttrReleaseThreshold, &keep)) != cudaSuccess ||
-      (e = cudaMemPoolSetAttribute(ctx->stage_pool, cudaMemPoolReuseAllowInternalDependencies, &no)) !=
-          cudaSuccess ||
-      (e = cudaEventCreateWithFlags(&ctx->staged, cudaEventDisableTiming)) != cudaSuccess)
+  cudaError_t e = cudaMemPoolCreate(&pool, &props);
+  if (e == cudaSuccess) e = cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+  if (e == cudaSuccess) e = cudaMemPoolSetAttribute(pool, cudaMemPoolReuseAllowInternalDependencies, &no);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking);
+  if (e != cudaSuccess) {   // nothing half-made is kept
+    if (st) cudaStreamDestroy(st);
+    if (ev) cudaEventDestroy(ev);
+    if (pool) cudaMemPoolDestroy(pool);
     return e;
-  return cudaStreamCreateWithFlags(&ctx->copy_in, cudaStreamNonBlocking);
+  }
+  ctx->stage_pool = pool;
+  ctx->staged = ev;
+  ctx->copy_in = st;
+  return cudaSuccess;
 }
 
 // Take a mark on `stream` for the bytes staged since the last one, then let
