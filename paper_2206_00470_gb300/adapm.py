@@ -191,7 +191,13 @@ def poisson_quantile(lam, p):
 
 
 class ParameterManager:
-    """One adapm context.  Device arrays are used in place; host arrays are copied."""
+    """One adapm context (adapm_create).  Device arrays are used in place; host arrays are copied.
+
+    relocate        move a key to its only worker with active intent instead of replicating it (Sec. 4.1)
+    action_timing   "start" (act when an intent becomes active), "adaptive" (Algorithm 1 at each sync, with
+                    timing_alpha / timing_p / timing_lambda0, 0 = the paper's 0.1 / 0.9999 / 10) or "signal"
+    delta_refresh   versioned refresh: sync leaves a sole holder's value when nobody else wrote the key
+    """
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
                  stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
