@@ -876,11 +876,29 @@ def oracle_sample(workload, budget_s, args):
     raise ValueError(workload)
 
 
+def host_cpu():
+    """The host CPU the oracle ran on: machine, model (from /proc/cpuinfo when it names one) and core count."""
+    import platform
+    model = None
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                key = ln.split(":")[0].strip().lower()
+                if key in ("model name", "cpu model", "hardware") and ":" in ln:
+                    model = ln.split(":", 1)[1].strip()
+                    break
+                if key == "cpu part" and model is None:
+                    model = "CPU part " + ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return {"machine": platform.machine(), "model": model, "nproc": os.cpu_count()}
+
+
 def cpu_baseline(args):
     threads = torch.get_num_threads()
     v, s, desc = oracle_sample(args.workload, args.cpu_budget, args)
     return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
-            "samples_per_s": s, "host_threads_available": threads}
+            "samples_per_s": s, "host_threads_available": threads, "host": host_cpu()}
 
 
 def run_reference(args, ws, rank):
