@@ -26,7 +26,9 @@ Fig. 10a, the owner recomputed by brute force from the call log, the
 Poisson quantile against scipy's, the rate estimate against the closed form
 of its recursion, the versioned refresh equal to the full one in exact
 arithmetic, the
-single-worker reduction to textbook mini-batch SGD,
+single-worker reduction to textbook mini-batch SGD and to textbook mini-batch
+AdaGrad, one AdaGrad step per occurrence of a repeated key (hand numbers and
+per-occurrence finite differences),
 fp64 finite-difference gradients, ComplEx scores by complex arithmetic and
 closed forms, Zipf frequencies by chi-square.  No function here is "parity
 unpinned".

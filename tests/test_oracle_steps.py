@@ -5,8 +5,15 @@
   and its DistMult special case (all-real rows);
 * closed forms: zero vectors give softplus(0) = log 2 per score; the AdaGrad
   delta on hand numbers;
-* a single worker with sync every clock reproduces textbook mini-batch SGD;
+* a single worker with sync every clock reproduces textbook mini-batch SGD, and with
+  AdaGrad a textbook mini-batch AdaGrad loop (the large MF configuration's path);
+* keys repeated inside one batch take one AdaGrad step per occurrence (MF on hand numbers,
+  ComplEx against per-occurrence finite differences), told apart from summing first;
 * MF loss falls on the tiny planted-rank workload.
+
+Planted mistakes in a scratch copy of the oracle's MF step were caught: swapping the
+row and column accumulators fails the textbook AdaGrad loop; dropping the g*g half of the
+delta row, or summing a key's gradients before one AdaGrad step, fails both MF pins.
 """
 import math
 
@@ -243,3 +250,125 @@ def test_sgns_step_pushes_sgd_deltas_of_the_batch_gradient():
     assert math.isclose(loss, batch_loss(x0), rel_tol=1e-9)
     g = fd_grad(batch_loss, x0)
     assert np.allclose(pm.main, x0 - lr * g, rtol=1e-5, atol=1e-7)
+
+
+# ---------------------------------------------------------------------------
+# AdaGrad (App. C: "SGD with AdaGrad"): the MF branch and repeated keys
+# ---------------------------------------------------------------------------
+
+def _textbook_minibatch_adagrad_mf(theta, acc, rank, batches, lr, eps):
+    """Mini-batch AdaGrad on 1/2 (v - u.w)^2 with a single store (no parameter manager).
+
+    theta [K, rank] factors, acc [K, rank] squared-gradient accumulators, fp64.
+    Every cell of a batch reads the store as it was at the start of the batch;
+    each occurrence of a factor row in a cell takes its own AdaGrad step
+    against the accumulator read at the start of the batch:
+        a_occ = acc[k] + g^2,  theta[k] -= lr g / sqrt(a_occ + eps),  acc[k] += g^2.
+    """
+    theta = theta.astype(np.float64).copy()
+    acc = acc.astype(np.float64).copy()
+    for rows, cols, vals in batches:
+        th0, ac0 = theta.copy(), acc.copy()
+        for i in range(len(rows)):
+            u, w = int(rows[i]), int(cols[i])
+            e = float(vals[i]) - float(th0[u] @ th0[w])
+            for k, g in ((u, -e * th0[w]), (w, -e * th0[u])):
+                theta[k] -= lr * g / np.sqrt(ac0[k] + g * g + eps)
+                acc[k] += g * g
+    return theta, acc
+
+
+def test_single_worker_adagrad_equals_textbook_minibatch_adagrad():
+    """The MF step with AdaGrad (the large MF configuration's path), one worker, sync every clock:
+    the manager's result equals a plain AdaGrad loop over the same batches.  Swapping the
+    accumulators of the row and column factor (or dropping the g*g half of the delta row) moves
+    the result by O(1) relative and fails this test (checked on a scratch copy of the oracle)."""
+    import dataclasses
+    cfg = dataclasses.replace(wl.TINY_MF, workers=1, epochs=1, adagrad=True, rank=8, lr=0.05)
+    data = wl.tiny_mf_dataset(cfg)
+    nclk = 25
+    init = init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
+    assert init.shape[1] == 2 * cfg.rank and not init[:, cfg.rank:].any()   # accumulators start at 0
+    # a non-zero starting accumulator so that a swapped or misplaced accumulator cannot go unnoticed
+    rng = np.random.default_rng(21)
+    init[:, cfg.rank:] = rng.uniform(0.01, 0.5, size=(cfg.num_keys, cfg.rank)).astype(np.float32)
+    pm = ParameterManagerOracle(cfg.num_keys, cfg.value_len, 1, init)
+    batches = [tuple(x.numpy() for x in wl.tiny_mf_batch(cfg, data, 0, c)) for c in range(nclk + 3)]
+
+    def keys_of(w, c):
+        return np.concatenate(batches[c][:2])
+
+    def work(w, c):
+        r, co, v = batches[c]
+        return steps.mf_step(pm, w, r, co, v, cfg.rank, cfg.lr, True, cfg.eps)
+
+    driver.start(pm, 1, cfg.lookahead, cfg.span, keys_of)
+    for c in range(nclk):
+        driver.clock(pm, 1, cfg.lookahead, cfg.span, c, keys_of, work)
+    th, ac = _textbook_minibatch_adagrad_mf(init[:, :cfg.rank], init[:, cfg.rank:], cfg.rank,
+                                            [batches[c] for c in range(nclk)], cfg.lr, cfg.eps)
+    # the manager stores fp32 after every clock; the textbook loop keeps fp64
+    assert np.allclose(pm.main[:, :cfg.rank], th, rtol=1e-5, atol=1e-6)
+    assert np.allclose(pm.main[:, cfg.rank:], ac, rtol=1e-5, atol=1e-6)
+    assert not np.allclose(pm.main[:, :cfg.rank], init[:, :cfg.rank], atol=1e-3)
+
+
+def test_mf_adagrad_repeated_key_takes_one_step_per_occurrence():
+    """Hand numbers, rank 1, eps 0, lr 1/2: row u = 1 meets columns w1 = 2 and w2 = -1 (values 0).
+    e1 = -2, e2 = 1; the row's gradients per occurrence are 4 and 1, the columns' 2 and -1.
+    Per occurrence: theta_u += -1/2 (4/sqrt(16) + 1/sqrt(1)) = -1, a_u += 16 + 1 = 17.
+    (Summing first would give theta_u += -1/2 * 5/sqrt(25) = -1/2 and a_u += 25.)"""
+    init = np.array([[1.0, 0.0], [2.0, 0.0], [-1.0, 0.0]], np.float32)   # [theta | a] of u, w1, w2
+    pm = ParameterManagerOracle(3, 2, 1, init)                          # no intents: pushes go to main
+    loss = steps.mf_step(pm, 0, np.array([0, 0]), np.array([1, 2]), np.array([0.0, 0.0], np.float32),
+                         1, 0.5, True, 0.0)
+    assert loss == 2.5
+    assert np.array_equal(pm.main, np.array([[0.0, 17.0], [1.5, 4.0], [-0.5, 1.0]], np.float32))
+
+
+def test_complex_adagrad_repeated_keys_take_one_step_per_occurrence():
+    """ComplEx with keys repeated inside one batch (a relation in both triples, an entity that is the
+    head of one triple and a negative tail of the other): every row occurrence takes its own AdaGrad
+    step with its own gradient, which is found here by fp64 finite differences of the batch loss with
+    respect to that occurrence alone (each occurrence made a variable of its own)."""
+    m, K = 2, 8
+    td = 2 * m
+    rng = np.random.default_rng(41)
+    init = np.zeros((K, 2 * td), np.float32)
+    init[:, :td] = rng.normal(0, 0.7, size=(K, td))
+    init[:, td:] = rng.uniform(0.05, 0.5, size=(K, td))
+    heads, rels, tails = [0, 1], [6, 6], [2, 3]
+    negs = [[4, 1], [0, 4]]                      # entity 1: head of triple 1 and a negative of triple 0
+    lr, eps = 0.1, 1e-8
+    pm = ParameterManagerOracle(K, 2 * td, 1, init)
+    steps.complex_step(pm, 0, heads, rels, tails, negs, td, lr, eps)
+
+    occ = heads + rels + tails + [k for row in negs for k in row]      # the step's row occurrences
+    x0 = init[occ, :td].astype(np.float64)                             # one variable per occurrence
+    n, k = len(heads), len(negs[0])
+
+    def loss_of(x):
+        total = 0.0
+        for i in range(n):
+            h, r, t = x[i], x[n + i], x[2 * n + i]
+            z = lambda a, b, c: sum(complex(a[q], a[m + q]) * complex(b[q], b[m + q]) *  # noqa: E731
+                                    complex(c[q], -c[m + q]) for q in range(m)).real
+            total += math.log1p(math.exp(-z(h, r, t)))
+            for j in range(k):
+                total += math.log1p(math.exp(z(h, r, x[3 * n + i * k + j])))
+        return total
+
+    g = fd_grad(loss_of, x0)
+    acc0 = init[occ, td:].astype(np.float64)
+    want = init.astype(np.float64).copy()
+    for o, key in enumerate(occ):
+        want[key, :td] += -lr * g[o] / np.sqrt(acc0[o] + g[o] * g[o] + eps)
+        want[key, td:] += g[o] * g[o]
+    assert np.allclose(pm.main, want, rtol=1e-5, atol=1e-7)
+    # the alternative reading (sum a key's gradients, then one AdaGrad step) is told apart
+    alt = init.astype(np.float64).copy()
+    for key in set(occ):
+        gs = sum(g[o] for o in range(len(occ)) if occ[o] == key)
+        alt[key, :td] += -lr * gs / np.sqrt(init[key, td:] + gs * gs + eps)
+        alt[key, td:] += gs * gs
+    assert not np.allclose(alt, want, rtol=1e-5, atol=1e-7)
