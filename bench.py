@@ -15,8 +15,12 @@ Reported (one JSON line on rank 0): pulled + pushed keys/s (value), training
 samples/s, per-operation device time and algorithmic GB/s, the roofline of
 the dominant kernel against the measured HBM copy peak, the end-to-end rate
 through the C ABI with pinned host buffers (host<->device copies timed), the
-CPU oracle's rate on a bounded sample, SM clocks sampled during the timed
-region, and the number of library kernels launched in it.
+CPU oracle's rate on a bounded sample (one thread), SM clocks sampled during
+the timed region, and the number of library kernels launched in it.  With the
+MF workload (the default) the same line carries a `micro` record: the
+parameter-access microbenchmark (100M keys x 64 floats, 2^20 Zipf(1.1) keys
+per worker and clock, span 1) measured the same way, with pull, push and sync
+against the HBM roofline (--micro-zipf adds other exponents as `micro_sweep`).
 
 With --gpus N > 1 (torchrun) every rank runs an independent replica of the
 workload on its own GPU: the path has no exchange step (replicas only).
@@ -33,6 +37,13 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
+
+# The CPU oracle baseline is a one-core figure: numpy's BLAS and OpenMP pools are held to one thread
+# (set before numpy is imported; the GPU path does no numerical work on the host).
+ORACLE_THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS",
+                      "VECLIB_MAXIMUM_THREADS", "NUMEXPR_NUM_THREADS")
+for _v in ORACLE_THREAD_VARS:
+    os.environ[_v] = "1"
 
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
@@ -583,11 +594,12 @@ def manager_options(args):
             "refresh": "versioned" if args.delta_refresh else "full"}
 
 
-def run_ours(args, ws, rank, local):
+def run_ours(args, ws, rank, local, workload=None):
     from paper_2206_00470_gb300 import adapm
+    workload = workload or args.workload
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
-    wk = WORKLOADS[args.workload](args, device)
+    wk = WORKLOADS[workload](args, device)
     total_clocks = args.warmup + args.steps
     t0 = time.time()
     wk.prepare(total_clocks + 2 * args.steps + 2)
@@ -684,7 +696,7 @@ def run_ours(args, ws, rank, local):
         traffic = None
         if name == "push_kernel":
             rows = (s1["push_rows"] - s0["push_rows"]) / steps / calls
-            traffic = recorded_traffic(args.workload, rows)
+            traffic = recorded_traffic(workload, rows)
         roofline = {"bound": "hbm", "kernel": name, "achieved": ach, "peak": peak,
                     "peak_source": peak_src, "unit": "GB/s", "frac": ach / peak,
                     "traffic": traffic, "alg_bytes_per_launch": a, "launch_ms": t_ms / calls}
@@ -896,9 +908,15 @@ def host_cpu():
 
 def cpu_baseline(args):
     threads = torch.get_num_threads()
-    v, s, desc = oracle_sample(args.workload, args.cpu_budget, args)
+    torch.set_num_threads(1)              # the oracle's batch generators run on the host too
+    try:
+        v, s, desc = oracle_sample(args.workload, args.cpu_budget, args)
+    finally:
+        torch.set_num_threads(threads)
     return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
-            "samples_per_s": s, "host_threads_available": threads, "host": host_cpu()}
+            "samples_per_s": s, "host_threads_available": os.cpu_count(),
+            "threads": {"torch": 1, **{k: os.environ.get(k) for k in ORACLE_THREAD_VARS}},
+            "host": host_cpu()}
 
 
 def run_reference(args, ws, rank):
@@ -910,11 +928,24 @@ def run_reference(args, ws, rank):
         "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": dict(WORKLOADS[args.workload](args, None).config(), parallelism="replicas1",
-                       **manager_options(args), reference="CPU oracle (plain Python/numpy, 1 core)"),
+                       **manager_options(args), l2="inputs larger than L2 (no flush)"),
+        "reference_kind": "CPU oracle (plain Python/numpy, 1 core)",
         "cpu_baseline": base,
         "e2e": {"value": base["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     return line
+
+
+MICRO_KEYS = ("value", "unit", "ms_per_step", "config", "gpu_launches", "clocks", "roofline", "ops", "e2e",
+              "stats", "replica_events_per_step", "setup_s")
+
+
+def micro_args(args, zipf):
+    """The microbenchmark's default shape (B = 2^20 keys per worker and clock, span 1, 100M keys) at
+    Zipf exponent `zipf`, with the run's steps, warm-up and manager options."""
+    a = argparse.Namespace(**vars(args))
+    a.workload, a.batch, a.zipf, a.span, a.keys = "micro", None, zipf, None, None
+    return a
 
 
 def main():
@@ -930,6 +961,10 @@ def main():
     ap.add_argument("--keys", type=int, default=None, help="micro: key-space size (default 1e8)")
     ap.add_argument("--mf-rows", type=int, default=None, help="mf: rows (default 10M)")
     ap.add_argument("--mf-cols", type=int, default=None, help="mf: columns (default 1M)")
+    ap.add_argument("--micro-zipf", type=lambda x: [float(v) for v in x.split(",") if v], default=[1.1],
+                    help="with the MF workload, also run the 100M-key microbenchmark at these Zipf exponents "
+                         "(comma-separated; the first is reported as 'micro', the rest as 'micro_sweep'; "
+                         "empty string: none)")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -956,6 +991,17 @@ def main():
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         base = cpu_baseline(args)
     line = run_ours(args, ws, rank, local)
+    if args.workload == "mf" and args.micro_zipf:
+        # the parameter-access microbenchmark (100M keys x 64 floats, 2^20 Zipf keys per worker and
+        # clock, span 1) in the same run: pull, push and sync against the HBM roofline
+        sweep = []
+        for z in args.micro_zipf:
+            torch.cuda.empty_cache()          # the library allocates with cudaMalloc, not torch's cache
+            rec = run_ours(micro_args(args, z), ws, rank, local, "micro")
+            sweep.append({k: rec[k] for k in MICRO_KEYS if k in rec})
+        line["micro"] = sweep[0]
+        if len(sweep) > 1:
+            line["micro_sweep"] = sweep[1:]
     if rank == 0:
         line["cpu_baseline"] = base
         print(json.dumps(line), flush=True)

@@ -181,7 +181,10 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
  *     cudaGetSymbolAddress; make that first call before any stream capture.
  *   - Every call (all contexts of the process) shares the one array: calls
  *     that overlap on the GPU (different streams, different contexts) race.
- *   - It allocates nothing: no cudaMalloc, cudaFree or pool allocation. */
+ *   - It allocates nothing: no cudaMalloc, cudaFree or pool allocation.
+ *   - Errors and profiling as adapm_push: a CUDA error returns ADAPM_ECUDA
+ *     and leaves the context unusable; with adapm_profile_enable on, its
+ *     time is recorded under operations 3 (push) and 6 (scatter kernels). */
 adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                                 const float* deltas);
 

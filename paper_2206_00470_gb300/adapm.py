@@ -282,6 +282,11 @@ class ParameterManager:
             raise ValueError("deltas must hold len(keys) * value_len floats")
         self._check(self._lib.adapm_push_noalloc(self._h, worker, k.ptr, k.n, d.ptr))
 
+    def last_error(self):
+        """adapm_last_error: the message of the last error returned on this context ("" if none)."""
+        msg = self._lib.adapm_last_error(self._h)
+        return msg.decode() if msg else ""
+
     def debug_fail_next_barrier(self):
         """Test hook: the next push's sort gives up its grid-barrier wait (ADAPM_ETIMEOUT at wait)."""
         self._check(self._lib.adapm_debug_fail_next_barrier(self._h))

@@ -275,31 +275,22 @@ cudaError_t finish_out(adapm_ctx* ctx, Output<T>* o) {
   return e;
 }
 
-struct ProfScope {
-  adapm_ctx* ctx;
-  int op;
-  cudaEvent_t a = nullptr, b = nullptr;
-  ProfScope(adapm_ctx* c, int o) : ctx(c), op(o) {
-    if (!ctx->prof) return;
-    a = take();
-    b = take();
-    if (a) cudaEventRecord(a, ctx->stream);
-  }
-  cudaEvent_t take() {
-    if (!ctx->spare_events.empty()) {
-      cudaEvent_t e = ctx->spare_events.back();
-      ctx->spare_events.pop_back();
-      return e;
-    }
-    cudaEvent_t e = nullptr;
-    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+cudaEvent_t take_prof_event(adapm_ctx* ctx) {
+  if (!ctx->spare_events.empty()) {
+    cudaEvent_t e = ctx->spare_events.back();
+    ctx->spare_events.pop_back();
     return e;
   }
-  ~ProfScope() {
-    if (!a || !b) return;
-    cudaEventRecord(b, ctx->stream);
-    ctx->pending.emplace_back(op, a, b);
-  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+struct ProfScope {
+  adapm_ctx* ctx;
+  ProfToken t;
+  ProfScope(adapm_ctx* c, int o) : ctx(c) { t = ctx_prof_start(ctx, o); }
+  ~ProfScope() { ctx_prof_stop(ctx, t); }
 };
 
 adapm_status check_launch(adapm_ctx* ctx, const char* where) {
@@ -443,6 +434,32 @@ void adapm::ctx_set_error(adapm_ctx* ctx, const char* msg) {
 
 void adapm::ctx_add_push_rows(adapm_ctx* ctx, uint64_t n) {
   if (ctx) ctx->push_rows_host += n;
+}
+
+int adapm::ctx_begin(adapm_ctx* ctx) { return check_ctx(ctx); }
+
+int adapm::ctx_fail_cuda(adapm_ctx* ctx, cudaError_t e, const char* where) { return cuda_fail(ctx, e, where); }
+
+ProfToken adapm::ctx_prof_start(adapm_ctx* ctx, int op) {
+  ProfToken t;
+  if (!ctx || !ctx->prof) return t;
+  t.op = op;
+  t.a = take_prof_event(ctx);
+  t.b = take_prof_event(ctx);
+  if (t.a) cudaEventRecord(t.a, ctx->stream);
+  return t;
+}
+
+void adapm::ctx_prof_stop(adapm_ctx* ctx, ProfToken& t) {
+  if (!ctx || t.op < 0) return;
+  if (t.a && t.b) {
+    cudaEventRecord(t.b, ctx->stream);
+    ctx->pending.emplace_back(t.op, t.a, t.b);
+  } else {   // an event could not be made: give back the one that was
+    if (t.a) ctx->spare_events.push_back(t.a);
+    if (t.b) ctx->spare_events.push_back(t.b);
+  }
+  t = ProfToken{};
 }
 
 extern "C" {

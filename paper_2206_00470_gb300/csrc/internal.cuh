@@ -143,5 +143,20 @@ struct CtxView {
 bool ctx_view(struct ::adapm_ctx* ctx, CtxView* out);
 void ctx_set_error(struct ::adapm_ctx* ctx, const char* msg);
 void ctx_add_push_rows(struct ::adapm_ctx* ctx, uint64_t n);
+// The checks every entry point starts with: a live context (ADAPM_EINVAL for
+// null, ADAPM_ECUDA once it is unusable), its last error cleared, its device
+// current.  Returns an adapm_status value (0 = ADAPM_OK).
+int ctx_begin(struct ::adapm_ctx* ctx);
+// A CUDA runtime error: records "where: message", marks the context unusable
+// (as every entry point does) and returns ADAPM_ECUDA.
+int ctx_fail_cuda(struct ::adapm_ctx* ctx, cudaError_t e, const char* where);
+// Per-operation timing (adapm_profile_enable): events recorded around an
+// operation's work on the context's stream; a no-op while profiling is off.
+struct ProfToken {
+  int op = -1;
+  cudaEvent_t a = nullptr, b = nullptr;
+};
+ProfToken ctx_prof_start(struct ::adapm_ctx* ctx, int op);
+void ctx_prof_stop(struct ::adapm_ctx* ctx, ProfToken& t);
 
 }  // namespace adapm

@@ -86,17 +86,25 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   return L;
 }
 
+// Profiling of one noalloc push: the same operations as adapm_push (3: the
+// whole push, 6: the scatter kernels), stopped on every path out.
+struct ProfGuard {
+  adapm_ctx* ctx;
+  adapm::ProfToken t;
+  ProfGuard(adapm_ctx* c, int op) : ctx(c) { t = adapm::ctx_prof_start(ctx, op); }
+  ~ProfGuard() { adapm::ctx_prof_stop(ctx, t); }
+};
+
 }  // namespace
 
 extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
                                            uint64_t n, const float* deltas) {
   using namespace adapm;
+  // a live context, its last error cleared, its device current
+  const adapm_status st = static_cast<adapm_status>(ctx_begin(ctx));
+  if (st != ADAPM_OK) return st;
   CtxView v;
   if (!ctx_view(ctx, &v)) return ADAPM_EINVAL;
-  if (v.broken) {
-    ctx_set_error(ctx, "context unusable after an earlier CUDA error");
-    return ADAPM_ECUDA;
-  }
   if (worker >= v.s.W) {
     ctx_set_error(ctx, "worker out of range");
     return ADAPM_EINVAL;
@@ -105,10 +113,6 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
   if (!keys || !deltas || n > (1ull << 31)) {
     ctx_set_error(ctx, "bad pointers/n");
     return ADAPM_EINVAL;
-  }
-  if (cudaSetDevice(v.device) != cudaSuccess) {
-    ctx_set_error(ctx, "cudaSetDevice failed");
-    return ADAPM_ECUDA;
   }
   if (!is_device_ptr(keys) || !is_device_ptr(deltas)) {
     ctx_set_error(ctx, "adapm_push_noalloc takes device arrays only");
@@ -129,22 +133,17 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
   }
   unsigned char* base = nullptr;
   cudaError_t e = scratch_for(v.device, &base);
-  if (e != cudaSuccess) {
-    ctx_set_error(ctx, cudaGetErrorString(e));
-    return ADAPM_ECUDA;
-  }
+  if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "cudaGetSymbolAddress"));
   auto at = [&](size_t off) { return reinterpret_cast<uint32_t*>(base + off); };
   uint32_t* longs = at(L.longs);
-  ctx_add_push_rows(ctx, n);
+  ProfGuard whole(ctx, 3);
   uint32_t *sk = nullptr, *sp = nullptr;
   // the array keeps the previous call's contents: the sort clears the
   // hot-key list count (and the distinct-key counter)
   e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist), v.sms,
                 v.dstate, v.bar_base, longs, &v.dstate->last_unique, v.stream, &sk, &sp);
-  if (e != cudaSuccess) {
-    ctx_set_error(ctx, cudaGetErrorString(e));
-    return ADAPM_ECUDA;
-  }
+  if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "push_noalloc sort"));
+  ctx_add_push_rows(ctx, n);
   PushArgs a{sk,
              sp,
              n,
@@ -157,11 +156,11 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
              longs + 1,
              longs,
              reinterpret_cast<float*>(base + L.lparts)};
-  launch_push(v.s, a, v.sms, v.stream);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) {
-    ctx_set_error(ctx, cudaGetErrorString(e));
-    return ADAPM_ECUDA;
+  {
+    ProfGuard scatter(ctx, 6);
+    launch_push(v.s, a, v.sms, v.stream);
   }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "push_noalloc scatter"));
   return ADAPM_OK;
 }
