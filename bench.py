@@ -585,13 +585,15 @@ def alg_bytes_per_step(wk, d, steps, relocate=False):
 
 
 COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "sync_refreshed", "created", "destroyed",
-            "relocations")
+            "relocations", "planned_pushes", "plan_misses")
 
 
 def manager_options(args):
-    """The parameter manager's placement, action timing and refresh options, as named in `config`."""
+    """The parameter manager's placement, action timing, refresh and push-plan options, as named in
+    `config`."""
     return {"placement": "relocate" if args.relocate else "replicate", "action_timing": args.timing,
-            "refresh": "versioned" if args.delta_refresh else "full"}
+            "refresh": "versioned" if args.delta_refresh else "full",
+            "push_plans": not getattr(args, "no_push_plans", False)}
 
 
 def run_ours(args, ws, rank, local, workload=None):
@@ -606,7 +608,7 @@ def run_ours(args, ws, rank, local, workload=None):
     init = wk.init_store()
     pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
                                 relocate=args.relocate, action_timing=args.timing,
-                                delta_refresh=args.delta_refresh)
+                                delta_refresh=args.delta_refresh, push_plans=not args.no_push_plans)
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -716,6 +718,7 @@ def run_ours(args, ws, rank, local, workload=None):
         # replica management per step (profiled pass): what relocation saves against always replicating
         "replica_events_per_step": {k: delta[k] / steps for k in ("created", "destroyed", "sync_replicas",
                                                                    "sync_refreshed", "sync_keys", "relocations")},
+        "push_plans_per_step": {k: delta[k] / steps for k in ("planned_pushes", "plan_misses")},
         "setup_s": setup_s,
     }
     if e2e_ms is not None:
@@ -937,7 +940,7 @@ def run_reference(args, ws, rank):
 
 
 MICRO_KEYS = ("value", "unit", "ms_per_step", "config", "gpu_launches", "clocks", "roofline", "ops", "e2e",
-              "stats", "replica_events_per_step", "setup_s")
+              "stats", "replica_events_per_step", "push_plans_per_step", "setup_s")
 
 
 def micro_args(args, zipf):
@@ -972,6 +975,8 @@ def main():
                     help="relocate a key to its only worker with active intent instead of always replicating")
     ap.add_argument("--delta-refresh", action="store_true",
                     help="versioned refresh: sync leaves a sole holder's value when nobody else wrote the key")
+    ap.add_argument("--no-push-plans", action="store_true",
+                    help="sort every push itself instead of using the sort made for its intent")
     ap.add_argument("--timing", default="start", choices=["start", "adaptive", "signal"],
                     help="act on an intent at its start clock, by Algorithm 1 at each sync, or when signalled")
     args = ap.parse_args()

@@ -84,6 +84,7 @@ typedef struct {
   double timing_lambda0;     /* ADAPM_ACT_ADAPTIVE: initial clocks per round, 0 = 10 */
   int32_t delta_refresh;     /* 0: sync refreshes every replica; 1: versioned refresh (see
                                 adapm_sync) */
+  int32_t no_push_plans;     /* 0: push plans (see adapm_intent) are made and used; 1: never */
 } adapm_config;
 
 /* Action timing (Sec. 4.2).
@@ -136,7 +137,19 @@ adapm_status adapm_destroy(adapm_ctx* ctx);
  * window that contains the current clock is active at once: missing
  * replicas are created before the call's work ends.  Otherwise the keys are
  * de-duplicated and stored until the worker's clock reaches clock_start.
- * Overlapping intents are reference-counted per (worker, key). */
+ * Overlapping intents are reference-counted per (worker, key).
+ *
+ * Push plans (unless no_push_plans).  An intent names the keys a worker
+ * will push, before it pushes them (a data loader signals a batch's keys
+ * when it builds the batch).  So the call also sorts its keys, with their
+ * positions, on a stream of the library's own that runs beside the library
+ * stream at low priority; the de-duplicated keys of a future window come
+ * from that sort.  A push (or training step) of the worker with as many keys
+ * as its newest intent whose window holds the current clock checks on the
+ * device that its keys equal that intent's, position by position, and then
+ * groups its rows by the stored sort instead of sorting again; otherwise it
+ * sorts.  Results are the same either way (the same stable order).
+ * adapm_wait also waits for that stream. */
 adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                           int64_t clock_start, int64_t clock_end);
 
@@ -283,6 +296,8 @@ typedef struct {
   uint64_t sync_replicas;    /* replicas refreshed by sync, cumulative */
   uint64_t relocations;      /* owner changes, cumulative (relocation only) */
   uint64_t sync_refreshed;   /* replica values written by sync, cumulative */
+  uint64_t planned_pushes;   /* pushes that checked a push plan (see adapm_intent), cumulative */
+  uint64_t plan_misses;      /* of those, pushes whose keys differed, so they sorted, cumulative */
 } adapm_stats;
 
 adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);

@@ -45,6 +45,7 @@ class Config(ctypes.Structure):
         ("timing_p", ctypes.c_double),
         ("timing_lambda0", ctypes.c_double),
         ("delta_refresh", ctypes.c_int32),
+        ("no_push_plans", ctypes.c_int32),
     ]
 
 
@@ -65,6 +66,8 @@ class Stats(ctypes.Structure):
         ("sync_replicas", ctypes.c_uint64),
         ("relocations", ctypes.c_uint64),
         ("sync_refreshed", ctypes.c_uint64),
+        ("planned_pushes", ctypes.c_uint64),
+        ("plan_misses", ctypes.c_uint64),
     ]
 
 
@@ -197,11 +200,13 @@ class ParameterManager:
     action_timing   "start" (act when an intent becomes active), "adaptive" (Algorithm 1 at each sync, with
                     timing_alpha / timing_p / timing_lambda0, 0 = the paper's 0.1 / 0.9999 / 10) or "signal"
     delta_refresh   versioned refresh: sync leaves a sole holder's value when nobody else wrote the key
+    push_plans      sort each intent's keys beside the library stream and let a push with the same keys
+                    use that sort (adapm_intent); False sorts every push itself
     """
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
                  stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
-                 timing_lambda0=0.0, delta_refresh=False):
+                 timing_lambda0=0.0, delta_refresh=False, push_plans=True):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -220,7 +225,8 @@ class ParameterManager:
         self.action_timing = action_timing
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
                      ctypes.c_void_p(handle), int(self.relocate), ACTION_TIMING[action_timing],
-                     float(timing_alpha), float(timing_p), float(timing_lambda0), int(bool(delta_refresh)))
+                     float(timing_alpha), float(timing_p), float(timing_lambda0), int(bool(delta_refresh)),
+                     int(not push_plans))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:

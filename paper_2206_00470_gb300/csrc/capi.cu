@@ -36,6 +36,16 @@ struct IntentList {
   uint32_t* keys = nullptr;   // device: cap distinct keys (no particular order), then the count word
   uint32_t* count = nullptr;
   uint64_t cap = 0;
+  // Push plan: the stable sort of the call's n keys with their positions
+  // (psk, psp), made on the plan stream; `ready` is recorded there after it
+  // (and after the distinct keys, when they come from the plan: from_plan).
+  uint32_t* psk = nullptr;
+  uint32_t* psp = nullptr;
+  uint64_t n = 0;
+  bool from_plan = false;
+  cudaEvent_t ready = nullptr;
+  void* in_owned = nullptr;   // the call's staged copy of host keys, read by the plan stream
+  int64_t start = 0, end = 0; // the window as signalled
 };
 
 struct WorkerState {
@@ -44,6 +54,7 @@ struct WorkerState {
   int64_t round_clock = 0;   // clock at the previous round
   std::map<int64_t, std::vector<int64_t>> starts;   // clock -> lists whose window opens
   std::map<int64_t, std::vector<int64_t>> ends;     // clock -> lists whose window closes
+  std::vector<int64_t> order;                       // recorded lists, oldest first
 };
 
 }  // namespace
@@ -85,6 +96,14 @@ struct adapm_ctx {
   std::vector<cudaEvent_t> spare_marks;
   uint64_t stage_unmarked = 0;   // bytes staged since the last mark
   uint64_t stage_live = 0;       // bytes staged since the oldest mark
+  // Push plans are sorted on plan_stream (lowest priority, so its blocks
+  // take what the library stream leaves), with scratch from plan_pool, which
+  // never makes one stream wait for the other on its own.
+  cudaStream_t plan_stream = nullptr;
+  cudaMemPool_t plan_pool = nullptr;
+  std::vector<cudaEvent_t> spare_ready;
+  uint32_t plan_seq = 0;
+  uint64_t planned_pushes = 0;
 };
 
 namespace {
@@ -157,6 +176,41 @@ cudaError_t ensure_copy_in(adapm_ctx* ctx) {
   ctx->staged = ev;
   ctx->copy_in = st;
   return cudaSuccess;
+}
+
+// The plan stream and its pool, made on the first intent that gets a plan.
+cudaError_t ensure_plan_stream(adapm_ctx* ctx) {
+  if (ctx->plan_stream) return cudaSuccess;
+  cudaMemPoolProps props{};
+  props.allocType = cudaMemAllocationTypePinned;
+  props.location.type = cudaMemLocationTypeDevice;
+  props.location.id = ctx->device;
+  cudaMemPool_t pool = nullptr;
+  cudaStream_t st = nullptr;
+  uint64_t keep = ~0ull;
+  int no = 0, least = 0, greatest = 0;
+  cudaError_t e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
+  if (e == cudaSuccess) e = cudaMemPoolCreate(&pool, &props);
+  if (e == cudaSuccess) e = cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+  if (e == cudaSuccess) e = cudaMemPoolSetAttribute(pool, cudaMemPoolReuseAllowInternalDependencies, &no);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&st, cudaStreamNonBlocking, least);
+  if (e != cudaSuccess) {
+    if (st) cudaStreamDestroy(st);
+    if (pool) cudaMemPoolDestroy(pool);
+    return e;
+  }
+  ctx->plan_pool = pool;
+  ctx->plan_stream = st;
+  return cudaSuccess;
+}
+
+cudaError_t take_ready_event(adapm_ctx* ctx, cudaEvent_t* ev) {
+  if (!ctx->spare_ready.empty()) {
+    *ev = ctx->spare_ready.back();
+    ctx->spare_ready.pop_back();
+    return cudaSuccess;
+  }
+  return cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
 }
 
 // Take a mark on `stream` for the bytes staged since the last one, then let
@@ -310,7 +364,9 @@ adapm_status check_ctx(adapm_ctx* ctx) {
 constexpr uint64_t kMaxN = 1ull << 31;
 
 // Refcount events of one worker -> destroy, then create replicas.
-adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventList>& ev) {
+adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventList>& ev,
+                          const std::vector<cudaEvent_t>& waits = {}) {
+  for (cudaEvent_t r : waits) CK(cudaStreamWaitEvent(ctx->stream, r, 0));
   uint64_t total = 0;
   for (const auto& e : ev) total += e.cap;
   if (total == 0) return ADAPM_OK;
@@ -329,10 +385,34 @@ adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventLis
 
 // Group, sum and apply n delta rows (device keys/rows); keys may hold kNoKey
 // when allow_nokey (rows the caller wants skipped).
+// The plan a push of n keys by worker w may use: the newest recorded intent
+// of w with n keys whose window (as signalled) holds the worker's clock.
+IntentList* find_plan(adapm_ctx* ctx, uint32_t w, uint64_t n) {
+  WorkerState& ws = ctx->workers[w];
+  for (auto it = ws.order.rbegin(); it != ws.order.rend(); ++it) {
+    IntentList& L = ctx->lists[*it];
+    if (L.psk && L.n == n && L.start <= ws.clock && ws.clock < L.end) return &L;
+  }
+  return nullptr;
+}
+
 adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint64_t n,
                          const float* drows, bool allow_nokey) {
   if (n == 0) return ADAPM_OK;
   uint32_t *ka = nullptr, *kb = nullptr, *va = nullptr, *vb = nullptr, *hist = nullptr;
+  IntentList* plan = find_plan(ctx, w, n);
+  uint32_t seq = 0;
+  if (plan) {
+    // check the plan on the device; the sort below runs only if it does not
+    // match (into this push's own arrays), and the scatter kernels read the
+    // plan's arrays or the sort's by the same check
+    CK(cudaStreamWaitEvent(ctx->stream, plan->ready, 0));
+    if (++ctx->plan_seq == 0) ctx->plan_seq = 1;
+    seq = ctx->plan_seq;
+    ctx->planned_pushes += 1;
+    launch_plan_verify(dkeys, plan->psk, plan->psp, n, ctx->s.K, allow_nokey, seq, &ctx->dstate->plan_miss,
+                       ctx->dstate, ctx->sms, ctx->stream);
+  }
   CK(pool_alloc(ctx, &ka, n));
   CK(pool_alloc(ctx, &kb, n));
   CK(pool_alloc(ctx, &va, n));
@@ -350,17 +430,23 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   // the sort also clears the hot-key list count and the distinct-key counter
   uint32_t *sk = nullptr, *sp = nullptr;
   CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
-               &ctx->bar_base, longs, &ctx->dstate->last_unique, ctx->stream, &sk, &sp));
+               &ctx->bar_base, longs, &ctx->dstate->last_unique, ctx->stream, &sk, &sp,
+               plan ? &ctx->dstate->plan_miss : nullptr, seq));
   ctx->push_rows_host += n;
   PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, longs + 1, longs, lparts};
+  if (plan) {
+    a.skeys = plan->psk;
+    a.spos = plan->psp;
+    a.alt_keys = sk;
+    a.alt_pos = sp;
+    a.plan_word = &ctx->dstate->plan_miss;
+    a.plan_seq = seq;
+  }
   {
     ProfScope ps(ctx, 6);
     launch_push(ctx->s, a, ctx->sms, ctx->stream);
   }
-  pool_free(ctx, ka);
-  pool_free(ctx, kb);
-  pool_free(ctx, va);
-  pool_free(ctx, vb);
+  for (uint32_t* p : {ka, kb, va, vb}) pool_free(ctx, p);
   pool_free(ctx, hist);
   pool_free(ctx, ph);
   pool_free(ctx, pt);
@@ -397,20 +483,73 @@ adapm_status act_in_round(adapm_ctx* ctx) {
     ws.round_clock = ws.clock;
     const int64_t bound = poisson_quantile(2.0 * std::max(ws.est, (double)delta), p);
     std::vector<EventList> ev;
+    std::vector<cudaEvent_t> waits;
     auto it = ws.starts.begin();
     while (it != ws.starts.end() && it->first < ws.clock + bound) {
       for (int64_t id : it->second) {
         const IntentList& L = ctx->lists[id];
         ev.push_back(EventList{L.keys, L.count, L.cap, +1});
+        if (L.from_plan) waits.push_back(L.ready);
       }
       it = ws.starts.erase(it);
     }
     if (!ev.empty()) {
-      const adapm_status st = apply_events(ctx, w, ev);
+      const adapm_status st = apply_events(ctx, w, ev, waits);
       if (st != ADAPM_OK) return st;
     }
   }
   return ADAPM_OK;
+}
+
+// Sort an intent's keys with their positions on the plan stream (a phased
+// sort: no block waits for another, so it runs in whatever the library
+// stream leaves of the GPU), into L.psk / L.psp; with from_plan the distinct
+// keys follow from the sorted ones (ascending) into L.keys / L.count.
+// L.ready is recorded on the plan stream after all of it.  The library
+// stream must have enqueued the keys (and L's arrays) before `after`.
+cudaError_t make_plan(adapm_ctx* ctx, IntentList& L, const uint32_t* keys, cudaEvent_t after) {
+  cudaError_t e = ensure_plan_stream(ctx);
+  if (e != cudaSuccess) return e;
+  cudaStream_t ps = ctx->plan_stream;
+  const uint64_t n = L.n;
+  if ((e = cudaStreamWaitEvent(ps, after, 0)) != cudaSuccess) return e;
+  uint32_t *tk = nullptr, *tv = nullptr, *hist = nullptr, *tmp = nullptr;
+  auto palloc = [&](uint32_t** p, size_t words) {
+    return cudaMallocFromPoolAsync(reinterpret_cast<void**>(p), (words ? words : 1) * sizeof(uint32_t),
+                                   ctx->plan_pool, ps);
+  };
+  if ((e = palloc(&tk, n)) != cudaSuccess || (e = palloc(&tv, n)) != cudaSuccess ||
+      (e = palloc(&hist, sort_scratch_words(n))) != cudaSuccess ||
+      (e = palloc(&tmp, compact_tmp_words(n))) != cudaSuccess)
+    return e;
+  const bool odd = sort_passes(ctx->bits) % 2 == 1;   // the sort ends in ka / va after odd passes
+  unsigned long long no_barriers = 0;
+  uint32_t *sk = nullptr, *sp = nullptr;
+  e = sort_keys(keys, n, ctx->s.K, false, ctx->bits, odd ? L.psk : tk, odd ? tk : L.psk, odd ? L.psp : tv,
+                odd ? tv : L.psp, hist, ctx->sms, ctx->dstate, &no_barriers, nullptr, nullptr, ps, &sk, &sp,
+                nullptr, 0, /*phased=*/true);
+  if (e != cudaSuccess) return e;
+  if (L.from_plan) compact_sorted_heads(L.psk, n, L.keys, L.count, tmp, ps);
+  for (uint32_t* p : {tk, tv, hist, tmp}) cudaFreeAsync(p, ps);
+  if ((e = take_ready_event(ctx, &L.ready)) != cudaSuccess) return e;
+  if ((e = cudaEventRecord(L.ready, ps)) != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+// Free an intent list whose window closed (on the library stream, after
+// its plan is complete).
+cudaError_t close_list(adapm_ctx* ctx, uint32_t w, int64_t id) {
+  IntentList& L = ctx->lists[id];
+  cudaError_t e = cudaSuccess;
+  if (L.ready) {
+    e = cudaStreamWaitEvent(ctx->stream, L.ready, 0);
+    ctx->spare_ready.push_back(L.ready);   // the wait has captured it; it can be recorded again
+  }
+  for (void* p : {(void*)L.keys, (void*)L.psk, (void*)L.psp, L.in_owned}) pool_free(ctx, p);
+  auto& order = ctx->workers[w].order;
+  order.erase(std::remove(order.begin(), order.end(), id), order.end());
+  ctx->lists.erase(id);
+  return e;
 }
 
 }  // namespace
@@ -553,7 +692,13 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   if (!ctx) return ADAPM_EINVAL;
   cudaSetDevice(ctx->device);
   if (ctx->stream) cudaStreamSynchronize(ctx->stream);
-  for (auto& kv : ctx->lists) cudaFree(kv.second.keys);
+  if (ctx->plan_stream) cudaStreamSynchronize(ctx->plan_stream);
+  for (auto& kv : ctx->lists) {
+    for (void* p : {(void*)kv.second.keys, (void*)kv.second.psk, (void*)kv.second.psp, kv.second.in_owned})
+      if (p) cudaFree(p);
+    if (kv.second.ready) cudaEventDestroy(kv.second.ready);
+  }
+  for (auto e : ctx->spare_ready) cudaEventDestroy(e);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
                   s.stamp, s.own, s.dirty, ctx->dstate};
@@ -570,6 +715,8 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   if (ctx->staged) cudaEventDestroy(ctx->staged);
   if (ctx->copy_in) cudaStreamDestroy(ctx->copy_in);
   if (ctx->stage_pool) cudaMemPoolDestroy(ctx->stage_pool);
+  if (ctx->plan_stream) cudaStreamDestroy(ctx->plan_stream);
+  if (ctx->plan_pool) cudaMemPoolDestroy(ctx->plan_pool);
   if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
   if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
   cudaGetLastError();
@@ -585,11 +732,17 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   if (n > kMaxN || (n > 0 && !keys)) return fail(ctx, ADAPM_EINVAL, "bad keys/n");
   WorkerState& ws = ctx->workers[worker];
   if (clock_end <= clock_start || clock_end <= ws.clock) return ADAPM_OK;   // never active
+  const int64_t signalled_start = clock_start;
   // acting on signal: the window starts now
   if (ctx->cfg.action_timing == ADAPM_ACT_ON_SIGNAL && clock_start > ws.clock) clock_start = ws.clock;
   ProfScope ps(ctx, 0);
   IntentList L;
   L.cap = n;
+  L.n = n;
+  L.start = signalled_start;
+  L.end = clock_end;
+  const bool now = clock_start <= ws.clock;   // the window contains the current clock: active at once
+  const bool plan = n > 0 && !ctx->cfg.no_push_plans;
   CK(cudaMallocFromPoolAsync((void**)&L.keys, (n + 1) * sizeof(uint32_t), ctx->pool, ctx->stream));
   L.count = L.keys + n;
   if (n == 0) {
@@ -597,18 +750,36 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   } else {
     Input<uint32_t> in;
     CK(stage_in(ctx, keys, n, &in));
-    if (++ctx->intent_tag == 0) {   // tags wrapped: clear the stamps
-      CK(cudaMemsetAsync(ctx->s.stamp, 0, ctx->s.K * 4, ctx->stream));
-      ctx->intent_tag = 1;
+    if (plan) {
+      CK(pool_alloc(ctx, &L.psk, n));
+      CK(pool_alloc(ctx, &L.psp, n));
     }
-    CK(cudaMemsetAsync(L.count, 0, sizeof(uint32_t), ctx->stream));
-    launch_intent_dedup(ctx->s, in.dev, n, ctx->intent_tag, L.keys, L.count, ctx->sms, ctx->stream);
-    pool_free(ctx, in.owned);
+    // a window that opens later takes its distinct keys from the plan; one
+    // that is active now needs them at once, from the hash-set pass here
+    L.from_plan = plan && !now;
+    if (!L.from_plan) {
+      if (++ctx->intent_tag == 0) {   // tags wrapped: clear the stamps
+        CK(cudaMemsetAsync(ctx->s.stamp, 0, ctx->s.K * 4, ctx->stream));
+        ctx->intent_tag = 1;
+      }
+      CK(cudaMemsetAsync(L.count, 0, sizeof(uint32_t), ctx->stream));
+      launch_intent_dedup(ctx->s, in.dev, n, ctx->intent_tag, L.keys, L.count, ctx->sms, ctx->stream);
+    }
+    if (plan) {
+      cudaEvent_t after = nullptr;
+      CK(take_ready_event(ctx, &after));
+      CK(cudaEventRecord(after, ctx->stream));
+      CK(make_plan(ctx, L, in.dev, after));
+      ctx->spare_ready.push_back(after);   // the plan stream's wait has captured it
+      L.in_owned = in.owned;               // freed when the list closes, after the plan
+    } else {
+      pool_free(ctx, in.owned);
+    }
   }
   const int64_t id = ctx->next_list++;
   ctx->lists[id] = L;
-  if (clock_start <= ws.clock) {
-    // the window contains the current clock: active at once
+  ws.order.push_back(id);
+  if (now) {
     st = apply_events(ctx, worker, {EventList{L.keys, L.count, L.cap, +1}});
     if (st != ADAPM_OK) return st;
   } else {
@@ -627,11 +798,13 @@ adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker) {
   const int64_t c = ws.clock;
   std::vector<EventList> ev;
   std::vector<int64_t> closing;
+  std::vector<cudaEvent_t> waits;   // plans that the opening lists' distinct keys come from
   auto it = ws.starts.find(c);
   if (it != ws.starts.end()) {
     for (int64_t id : it->second) {
       const IntentList& L = ctx->lists[id];
       ev.push_back(EventList{L.keys, L.count, L.cap, +1});
+      if (L.from_plan) waits.push_back(L.ready);
     }
     ws.starts.erase(it);
   }
@@ -646,11 +819,8 @@ adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker) {
   }
   if (ev.empty()) return ADAPM_OK;
   ProfScope ps(ctx, 1);
-  st = apply_events(ctx, worker, ev);
-  for (int64_t id : closing) {
-    pool_free(ctx, ctx->lists[id].keys);
-    ctx->lists.erase(id);
-  }
+  st = apply_events(ctx, worker, ev, waits);
+  for (int64_t id : closing) CK(close_list(ctx, worker, id));
   return st;
 }
 
@@ -734,6 +904,7 @@ adapm_status adapm_wait(adapm_ctx* ctx) {
   if (ctx->broken) return fail(ctx, ADAPM_ECUDA, "context unusable after an earlier CUDA error");
   cudaSetDevice(ctx->device);
   CK(cudaStreamSynchronize(ctx->stream));
+  if (ctx->plan_stream) CK(cudaStreamSynchronize(ctx->plan_stream));   // plans read the callers' keys
   uint32_t errors = 0;
   CK(cudaMemcpy(&errors, &ctx->dstate->errors, sizeof errors, cudaMemcpyDeviceToHost));
   if (errors) CK(cudaMemset(&ctx->dstate->errors, 0, sizeof errors));
@@ -1020,6 +1191,8 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
   out->sync_replicas = h.sync_replicas;
   out->relocations = h.relocations;
   out->sync_refreshed = h.sync_refreshed;
+  out->planned_pushes = ctx->planned_pushes;
+  out->plan_misses = h.plan_misses;
   return ADAPM_OK;
 }
 

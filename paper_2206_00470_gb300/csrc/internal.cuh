@@ -45,6 +45,8 @@ struct DevState {
   uint32_t n_create_ok;   // creates that got a slot
   uint32_t errors;        // ErrBits, sticky until read by adapm_wait
   uint32_t last_unique;   // distinct keys of the last push
+  uint32_t plan_miss;     // sequence number of the last push whose plan did not match its keys
+  uint32_t pad0;
   unsigned long long created;
   unsigned long long destroyed;
   int32_t live;
@@ -55,6 +57,7 @@ struct DevState {
   unsigned long long sync_replicas;   // replicas refreshed by sync (cumulative)
   unsigned long long relocations;     // owner changes (relocation mode, cumulative)
   unsigned long long sync_refreshed;  // replica values written by sync (cumulative)
+  unsigned long long plan_misses;     // pushes whose plan did not match their keys (cumulative)
   // grid barriers of the sort: blocks arrived, over the context's lifetime
   // (a line of its own, away from the counters above)
   alignas(128) unsigned long long bar_arrivals;
@@ -111,11 +114,34 @@ __device__ __forceinline__ bool sort_failed(const DevState* st) {
 // stream runs (counters of the consumer).  If a grid-barrier wait gives
 // up, the kernel sets ERR_TIMEOUT and returns; every kernel that consumes a
 // sort checks that bit first and does nothing while it is set.
+//
+// Plans: with plan_word non-null the launch sorts only if *plan_word ==
+// plan_seq when it runs (plan_verify stored a mismatch); otherwise its
+// blocks account their grid barriers and return, leaving ka/kb/va/vb as
+// they are (the caller's verified plan holds the result).
+// phased = true runs the sort as 1 + 2 * passes ordinary launches (kernel
+// boundaries instead of grid barriers, *bar_base untouched): for a stream
+// that runs beside other work, where a cooperative launch would wait for
+// the whole GPU.
 size_t sort_scratch_words(uint64_t n);
+int sort_passes(int bits);
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
                       DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
-                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out);
+                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out,
+                      const uint32_t* plan_word = nullptr, uint32_t plan_seq = 0, bool phased = false);
+
+// Checks a plan (sk, sp: the stable key sort of an earlier key list) against
+// the n keys of a push: stores seq in *word unless keys[sp[i]] == sk[i] for
+// every i (out-of-range keys matching the sentinel); sets ERR_KEY_RANGE for
+// an out-of-range push key as the sort would.
+void launch_plan_verify(const uint32_t* keys, const uint32_t* sk, const uint32_t* sp, uint64_t n, uint64_t K,
+                        bool allow_nokey, uint32_t seq, uint32_t* word, DevState* st, int sms,
+                        cudaStream_t stream);
+
+// The distinct valid keys of a sorted array, ascending, into out; count to *count.
+void compact_sorted_heads(const uint32_t* sk, uint64_t n, uint32_t* out, uint32_t* count, uint32_t* tmp,
+                          cudaStream_t stream);
 
 // Stream compaction (a count / scan / write pass), tmp of compact_tmp_words(n).
 size_t compact_tmp_words(uint64_t n);

@@ -130,6 +130,10 @@ struct SortArgs {
   uint32_t* clear0;              // words set to zero by the launch (nullptr: none)
   uint32_t* clear1;
   unsigned long long bar_base;   // st->bar_arrivals when the launch starts
+  const uint32_t* plan_word;     // with plan_seq != 0: the sort runs only if *plan_word == plan_seq
+  uint32_t plan_seq;
+  int phase;                     // -1: every phase, grid barriers between (cooperative launch);
+                                 // k >= 0: phase k alone (0 count, 1 + 2p scan, 2 + 2p scatter of pass p)
   int allow_nokey;
   int passes;
   int per;
@@ -251,7 +255,8 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   const int warp = threadIdx.x >> 5;
   const uint32_t B = gridDim.x;
   const uint32_t b = blockIdx.x;
-  if (b == 0 && threadIdx.x == 0) {
+  const bool coop = a.phase < 0;
+  if (b == 0 && threadIdx.x == 0 && (coop || a.phase == 0)) {
     if (a.clear0) *a.clear0 = 0u;
     if (a.clear1) *a.clear1 = 0u;
   }
@@ -259,6 +264,16 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
   __syncthreads();
   if (sm.abort) return;
+  // a verified plan already holds this sort's result: arrive at every barrier
+  // of the launch at once (the host counts them) and stop
+  if (a.plan_seq != 0u && ld_acquire(a.plan_word) != a.plan_seq) {
+    if (threadIdx.x == 0 && coop) {
+      const unsigned long long nb = sort_barriers(a.passes);
+      asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(&a.st->bar_arrivals), "l"(nb) : "memory");
+    }
+    return;
+  }
+  auto run = [&](int ph) { return coop || a.phase == ph; };
   uint32_t nbar = 0;
   const uint64_t chunk = (a.n + B - 1) / B;
   const uint64_t c0 = a.n < b * chunk ? a.n : b * chunk;
@@ -273,7 +288,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   uint32_t key[ITEMS], val[ITEMS], rank[ITEMS];
   bool bad = false;
   // 0. first pass digit counts of the chunk (ranks kept when one sub-tile)
-  {
+  if (run(0)) {
     const int nbits = a.per < a.bits ? a.per : a.bits;
     const uint32_t mask = (1u << nbits) - 1u;
     if (single) {
@@ -293,8 +308,8 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     }
     for (uint32_t d = threadIdx.x; d <= mask; d += kSortThreads) table0[(uint64_t)d * B + b] = sm.cnt[d];
     if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) set_error(a.st, ERR_KEY_RANGE);
-    if (!grid_barrier(a, nbar, sm)) return;
   }
+  if (coop && !grid_barrier(a, nbar, sm)) return;
   int shift = 0;
   for (int p = 0; p < a.passes; ++p) {
     const bool first = p == 0;
@@ -312,6 +327,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     // round of coalesced loads, combined through shared memory; otherwise
     // one warp per digit row, read in batches.  Every block
     // also clears its own column of the next pass's table.
+    if (run(1 + 2 * p)) {
     if (more)
       for (uint32_t d = threadIdx.x; d <= nmask; d += kSortThreads) tnext[(uint64_t)d * B + b] = 0u;
     if (B <= 16) {
@@ -398,9 +414,11 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
         if (lane == 0) a.totals[d] = carry;
       }
     }
-    if (!grid_barrier(a, nbar, sm)) return;
+    }   // scan phase
+    if (coop && !grid_barrier(a, nbar, sm)) return;
     // 2. scatter: digit bases, then the chunk's sub-tiles in order; each
     // written key is counted for the next pass in the chunk it lands in
+    if (run(2 + 2 * p)) {
     {
       uint32_t v[kDPT], local = 0;
 #pragma unroll
@@ -420,7 +438,8 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     }
     for (uint64_t s0 = c0; s0 < c1; s0 += SUB) {
       const uint64_t s1 = s0 + SUB < c1 ? s0 + SUB : c1;
-      if (!(single && first))
+      // (the first pass's ranks survive from the count only within one launch)
+      if (!(single && first && coop))
         load_rank<POS, ITEMS>(a, kin, vin, first, s0, s1, shift, nbits, key, val, rank, bad, sm);
       {
         uint32_t local = 0;
@@ -474,7 +493,8 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
       }
       __syncthreads();
     }
-    if (more) {
+    }   // scatter phase
+    if (coop && more) {
       if (!grid_barrier(a, nbar, sm)) return;
     }
     kin = kout;
@@ -492,6 +512,17 @@ struct MapSel {
   uint64_t n;
   __device__ bool flag(uint64_t i) const { return m[i] >= 0; }
   __device__ uint32_t value(uint64_t i) const { return (uint32_t)i; }
+};
+
+// the first copy of every valid key of a sorted array (the distinct keys, ascending)
+struct HeadSel {
+  const uint32_t* sk;
+  uint64_t n;
+  __device__ bool flag(uint64_t i) const {
+    const uint32_t k = sk[i];
+    return k != kNoKey && (i == 0 || sk[i - 1] != k);
+  }
+  __device__ uint32_t value(uint64_t i) const { return sk[i]; }
 };
 
 template <class Sel>
@@ -584,12 +615,58 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   if (B > kMaxSortBlocks) B = kMaxSortBlocks;
   if (B < 1) B = 1;
   a.bar_base = *bar_base;
+  a.phase = -1;
   void* params[] = {&a};
   note_launches(1);
   const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, ITEMS>, dim3((unsigned)B),
                                                     dim3(kSortThreads), params, 0, stream);
   if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes) * B;
   return e;
+}
+
+// The same sort as 1 + 2 * passes ordinary launches, one phase each: the
+// kernel boundaries are its barriers, so nothing waits on another block and
+// the blocks need not be resident together (for a stream that runs beside
+// other work).  B = one block per sub-tile of keys.
+template <bool POS, int ITEMS>
+cudaError_t launch_sort_phased(SortArgs& a, cudaStream_t stream) {
+  constexpr uint64_t SUB = (uint64_t)kSortThreads * ITEMS;
+  uint64_t B = (a.n + SUB - 1) / SUB;
+  if (B > kMaxSortBlocks) B = kMaxSortBlocks;
+  if (B < 1) B = 1;
+  a.bar_base = 0;
+  const int phases = 1 + 2 * a.passes;
+  note_launches((uint64_t)phases);
+  for (int ph = 0; ph < phases; ++ph) {
+    a.phase = ph;
+    sort_kernel<POS, ITEMS><<<(unsigned)B, kSortThreads, 0, stream>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+// Plan check of a push: for every sorted position i, the push's key at
+// position sp[i] must equal sk[i] (both out of range where sk[i] is the
+// sentinel).  Then (sk, sp) is exactly the stable key sort of the push's
+// keys, since sk is sorted and sp a permutation.  A mismatch anywhere
+// stores `seq` in *word.  Every push key is read once (sp is a
+// permutation), so out-of-range keys are reported here as the sort would.
+__global__ void __launch_bounds__(kSortThreads) plan_verify_kernel(const uint32_t* __restrict__ keys,
+                                                                   const uint32_t* __restrict__ sk,
+                                                                   const uint32_t* __restrict__ sp, uint64_t n,
+                                                                   uint64_t K, int allow_nokey, uint32_t seq,
+                                                                   uint32_t* word, DevState* st) {
+  bool bad = false, miss = false;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t s = __ldg(sk + i);
+    const uint32_t pos = __ldg(sp + i);
+    const uint32_t k = pos < n ? __ldg(keys + pos) : s ^ 1u;
+    if (k >= K && !(allow_nokey && k == kNoKey)) bad = true;
+    miss |= s == kNoKey ? k < K : k != s;
+  }
+  // the first warp to record this push's mismatch counts it
+  if (__any_sync(0xFFFFFFFFu, miss) && (threadIdx.x & 31) == 0 && atomicExch(word, seq) != seq)
+    atomicAdd(&st->plan_misses, 1ull);
+  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(st, ERR_KEY_RANGE);
 }
 
 }  // namespace
@@ -607,15 +684,21 @@ size_t sort_scratch_words(uint64_t n) {
   return (size_t)(kScratchHead + kDigits + 2 * rows * kDigits);   // totals, two tables
 }
 
+int sort_passes(int bits) { return plan_for(bits).passes; }
+
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
                       DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
-                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out) {
+                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out, const uint32_t* plan_word,
+                      uint32_t plan_seq, bool phased) {
   const PassPlan pl = plan_for(bits);
   if (keys_out) *keys_out = pl.passes % 2 ? ka : kb;
   if (pos_out) *pos_out = va ? (pl.passes % 2 ? va : vb) : nullptr;
   if (n == 0) return cudaSuccess;
   SortArgs a;
+  a.plan_word = plan_word;
+  a.plan_seq = plan_word ? plan_seq : 0u;
+  a.phase = -1;
   a.raw = raw;
   a.n = n;
   a.K = K;
@@ -634,9 +717,24 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
   a.bits = bits;
   // batches that would give fewer blocks than SMs take sub-tiles of half the
   // size: twice the blocks, half the ranking work per block
-  if ((n + kSub - 1) / kSub < (uint64_t)sms)
+  const bool small = (n + kSub - 1) / kSub < (uint64_t)sms;
+  if (phased) {
+    if (small) return va ? launch_sort_phased<true, 4>(a, stream) : launch_sort_phased<false, 4>(a, stream);
+    return va ? launch_sort_phased<true, kItems>(a, stream) : launch_sort_phased<false, kItems>(a, stream);
+  }
+  if (small)
     return va ? launch_sort<true, 4>(a, bar_base, sms, stream) : launch_sort<false, 4>(a, bar_base, sms, stream);
   return va ? launch_sort<true, kItems>(a, bar_base, sms, stream) : launch_sort<false, kItems>(a, bar_base, sms, stream);
+}
+
+void launch_plan_verify(const uint32_t* keys, const uint32_t* sk, const uint32_t* sp, uint64_t n, uint64_t K,
+                        bool allow_nokey, uint32_t seq, uint32_t* word, DevState* st, int sms, cudaStream_t stream) {
+  if (n == 0) return;
+  uint64_t b = (n + kSortThreads * 4 - 1) / (kSortThreads * 4);
+  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+  note_launches(1);
+  plan_verify_kernel<<<(unsigned)b, kSortThreads, 0, stream>>>(keys, sk, sp, n, K, allow_nokey ? 1 : 0, seq, word,
+                                                               st);
 }
 
 size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile + 1); }
@@ -644,6 +742,11 @@ size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile +
 void compact_replica_keys(const int32_t* map_w, uint64_t K, uint32_t* out, uint32_t* count,
                           uint32_t* tmp, cudaStream_t stream) {
   compact(MapSel{map_w, K}, out, count, tmp, stream);
+}
+
+void compact_sorted_heads(const uint32_t* sk, uint64_t n, uint32_t* out, uint32_t* count, uint32_t* tmp,
+                          cudaStream_t stream) {
+  compact(HeadSel{sk, n}, out, count, tmp, stream);
 }
 
 }  // namespace adapm

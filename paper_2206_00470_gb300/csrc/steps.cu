@@ -190,14 +190,16 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
   const uint32_t D4 = s.D >> 2;          // = 4 * h4: [theta re | theta im | a re | a im]
   const int32_t* mapw = s.map + (uint64_t)w * s.K;
   float4* d4 = reinterpret_cast<float4*>(o.drows);
-  const uint64_t per = 3 + (uint64_t)n_neg;
+  // delta rows in the order the keys of a batch are listed: all heads, all
+  // relations, all true tails, then the negatives triple by triple
+  const uint64_t rh = 0, rrel = n, rt = 2 * n, rneg = 3 * n;
   double lsum = 0.0;
   for (uint64_t i = warp; i < n; i += nwarps) {
-    const uint64_t base = i * per;
     const uint32_t kh = heads[i], kr = rels[i], kt = tails[i];
     if (kh >= s.K || kr >= s.K || kt >= s.K) {
       if (lane == 0) set_error(s.st, ERR_KEY_RANGE);
-      for (uint64_t q = lane; q < per; q += 32) o.dkeys[base + q] = kNoKey;
+      if (lane < 3) o.dkeys[(uint64_t)lane * n + i] = kNoKey;
+      for (uint64_t q = lane; q < n_neg; q += 32) o.dkeys[rneg + i * n_neg + q] = kNoKey;
       continue;
     }
     const float4* ph = row_ptr(s, mapw, kh);
@@ -272,7 +274,7 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
         const uint32_t j = j0 + u;
         const float phi = group_sum<32>(part[u]);
         if (j >= J) continue;
-        const uint64_t row = base + (j == 0 ? 2 : 2 + j);
+        const uint64_t row = j == 0 ? rt + i : rneg + i * n_neg + (j - 1);
         if (k0[u] == kNoKey) {
           if (lane == 0) o.dkeys[row] = kNoKey;
           continue;
@@ -316,18 +318,18 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
                                        hre[c].z * Tim[c].z - him[c].z * Tre[c].z, hre[c].w * Tim[c].w - him[c].w * Tre[c].w);
       const float4 ah_re = ph[2 * h4 + q], ah_im = ph[3 * h4 + q];
       const float4 ar_re = pr[2 * h4 + q], ar_im = pr[3 * h4 + q];
-      d4[base * D4 + q] = ada_theta4(gh_re, ah_re, lr, eps);
-      d4[base * D4 + h4 + q] = ada_theta4(gh_im, ah_im, lr, eps);
-      d4[base * D4 + 2 * h4 + q] = sq4(gh_re);
-      d4[base * D4 + 3 * h4 + q] = sq4(gh_im);
-      d4[(base + 1) * D4 + q] = ada_theta4(gr_re, ar_re, lr, eps);
-      d4[(base + 1) * D4 + h4 + q] = ada_theta4(gr_im, ar_im, lr, eps);
-      d4[(base + 1) * D4 + 2 * h4 + q] = sq4(gr_re);
-      d4[(base + 1) * D4 + 3 * h4 + q] = sq4(gr_im);
+      d4[(rh + i) * D4 + q] = ada_theta4(gh_re, ah_re, lr, eps);
+      d4[(rh + i) * D4 + h4 + q] = ada_theta4(gh_im, ah_im, lr, eps);
+      d4[(rh + i) * D4 + 2 * h4 + q] = sq4(gh_re);
+      d4[(rh + i) * D4 + 3 * h4 + q] = sq4(gh_im);
+      d4[(rrel + i) * D4 + q] = ada_theta4(gr_re, ar_re, lr, eps);
+      d4[(rrel + i) * D4 + h4 + q] = ada_theta4(gr_im, ar_im, lr, eps);
+      d4[(rrel + i) * D4 + 2 * h4 + q] = sq4(gr_re);
+      d4[(rrel + i) * D4 + 3 * h4 + q] = sq4(gr_im);
     }
     if (lane == 0) {
-      o.dkeys[base] = kh;
-      o.dkeys[base + 1] = kr;
+      o.dkeys[rh + i] = kh;
+      o.dkeys[rrel + i] = kr;
     }
   }
   block_loss(lsum, o.loss_part);

@@ -21,6 +21,13 @@ struct PushArgs {
   uint32_t* long_list;    // push_long_list_words(nchunks) - 1 words of scratch
   uint32_t* long_count;   // one word, zeroed by the caller
   float* long_parts;      // push_long_part_rows(nchunks) x D floats of scratch
+  // With plan_seq != 0, skeys / spos are a push plan and alt_keys / alt_pos
+  // the sort made in its place; the kernels take the latter when
+  // *plan_word == plan_seq (the plan did not match this push's keys).
+  const uint32_t* alt_keys = nullptr;
+  const uint32_t* alt_pos = nullptr;
+  const uint32_t* plan_word = nullptr;
+  uint32_t plan_seq = 0;
 };
 
 // Scratch sizes of the hot-key (long segment) combine for nchunks chunks.
