@@ -143,8 +143,8 @@ adapm_status adapm_destroy(adapm_ctx* ctx);
  * will push, before it pushes them (a data loader signals a batch's keys
  * when it builds the batch).  So the call also sorts its keys, with their
  * positions, on a stream of the library's own that runs beside the library
- * stream at low priority; the de-duplicated keys of a future window come
- * from that sort.  A push (or training step) of the worker with as many keys
+ * stream at low priority; the de-duplicated keys of a window that opens two
+ * or more clocks ahead come from that sort.  A push (or training step) of the worker with as many keys
  * as its newest intent whose window holds the current clock checks on the
  * device that its keys equal that intent's, position by position, and then
  * groups its rows by the stored sort instead of sorting again; otherwise it
@@ -188,8 +188,8 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
  *     (ADAPM_EINVAL otherwise).
  *   - A push whose sort and partial-sum buffers exceed the 16 MiB returns
  *     ADAPM_EINVAL with the sizes in adapm_last_error().  On a 152-SM GPU
- *     every n up to about 440k rows fits at value_len 64, 520k at 200 and
- *     300, 300k at 512 and 14k at 1024.
+ *     every n up to about 420k rows fits at value_len 64, 510k at 200 and
+ *     300, 280k at 512 and 14k at 1024.
  *   - The first call on a device looks up the array's device address with
  *     cudaGetSymbolAddress; make that first call before any stream capture.
  *   - Every call (all contexts of the process) shares the one array: calls

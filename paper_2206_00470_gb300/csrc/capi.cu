@@ -420,20 +420,17 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
-  float *ph = nullptr, *pt = nullptr;
-  uint32_t* longs = nullptr;
+  float *ph = nullptr, *pt = nullptr, *sparts = nullptr;
   CK(pool_alloc(ctx, &ph, nchunks * ctx->s.D));
   CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
-  float* lparts = nullptr;
-  CK(pool_alloc(ctx, &longs, push_long_list_words(nchunks)));
-  CK(pool_alloc(ctx, &lparts, push_long_part_rows(nchunks) * ctx->s.D));
-  // the sort also clears the hot-key list count and the distinct-key counter
+  CK(pool_alloc(ctx, &sparts, push_span_part_rows(nchunks) * ctx->s.D));
+  // the sort also clears the distinct-key counter
   uint32_t *sk = nullptr, *sp = nullptr;
   CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
-               &ctx->bar_base, longs, &ctx->dstate->last_unique, ctx->stream, &sk, &sp,
+               &ctx->bar_base, &ctx->dstate->last_unique, nullptr, ctx->stream, &sk, &sp,
                plan ? &ctx->dstate->plan_miss : nullptr, seq));
   ctx->push_rows_host += n;
-  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, longs + 1, longs, lparts};
+  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, sparts};
   if (plan) {
     a.skeys = plan->psk;
     a.spos = plan->psp;
@@ -450,8 +447,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   pool_free(ctx, hist);
   pool_free(ctx, ph);
   pool_free(ctx, pt);
-  pool_free(ctx, longs);
-  pool_free(ctx, lparts);
+  pool_free(ctx, sparts);
   return check_launch(ctx, "push");
 }
 
@@ -754,9 +750,11 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
       CK(pool_alloc(ctx, &L.psk, n));
       CK(pool_alloc(ctx, &L.psp, n));
     }
-    // a window that opens later takes its distinct keys from the plan; one
-    // that is active now needs them at once, from the hash-set pass here
-    L.from_plan = plan && !now;
+    // a window that opens two or more clocks ahead takes its distinct keys
+    // from the plan; one that opens at the next advance (or is active now)
+    // would wait there for the plan, so its keys come from the hash-set pass
+    // here, and the plan only serves the push a clock later
+    L.from_plan = plan && clock_start > ws.clock + 1;
     if (!L.from_plan) {
       if (++ctx->intent_tag == 0) {   // tags wrapped: clear the stamps
         CK(cudaMemsetAsync(ctx->s.stamp, 0, ctx->s.K * 4, ctx->stream));

@@ -59,7 +59,7 @@ bool is_device_ptr(const void* p) {
 
 // Byte offsets of the scratch regions of one push of n rows.
 struct Layout {
-  size_t ka, kb, va, vb, hist, ph, pt, longs, lparts, total;
+  size_t ka, kb, va, vb, hist, ph, pt, sparts, total;
   uint64_t chunk, nchunks;
 };
 
@@ -80,8 +80,7 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   L.hist = take(adapm::sort_scratch_words(n) * 4);
   L.ph = take(L.nchunks * D * 4);
   L.pt = take(L.nchunks * D * 4);
-  L.longs = take(adapm::push_long_list_words(L.nchunks) * 4);
-  L.lparts = take(adapm::push_long_part_rows(L.nchunks) * D * 4);
+  L.sparts = take(adapm::push_span_part_rows(L.nchunks) * D * 4);
   L.total = off;
   return L;
 }
@@ -135,13 +134,13 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
   cudaError_t e = scratch_for(v.device, &base);
   if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "cudaGetSymbolAddress"));
   auto at = [&](size_t off) { return reinterpret_cast<uint32_t*>(base + off); };
-  uint32_t* longs = at(L.longs);
   ProfGuard whole(ctx, 3);
   uint32_t *sk = nullptr, *sp = nullptr;
-  // the array keeps the previous call's contents: the sort clears the
-  // hot-key list count (and the distinct-key counter)
+  // the array keeps the previous call's contents: every scratch word is
+  // written before it is read, except the distinct-key counter, which the
+  // sort clears
   e = sort_keys(keys, n, v.s.K, false, v.bits, at(L.ka), at(L.kb), at(L.va), at(L.vb), at(L.hist), v.sms,
-                v.dstate, v.bar_base, longs, &v.dstate->last_unique, v.stream, &sk, &sp);
+                v.dstate, v.bar_base, &v.dstate->last_unique, nullptr, v.stream, &sk, &sp);
   if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "push_noalloc sort"));
   ctx_add_push_rows(ctx, n);
   PushArgs a{sk,
@@ -153,9 +152,7 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
              L.chunk,
              L.nchunks,
              worker,
-             longs + 1,
-             longs,
-             reinterpret_cast<float*>(base + L.lparts)};
+             reinterpret_cast<float*>(base + L.sparts)};
   {
     ProfGuard scatter(ctx, 6);
     launch_push(v.s, a, v.sms, v.stream);

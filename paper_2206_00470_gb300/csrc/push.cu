@@ -1,11 +1,12 @@
 // push: the rows of each distinct key of one call are summed and added to the
 // worker's replica (value and pending updates) or to main (Sec. 4,
-// App. B.1.2).  Sorted (key, position) pairs are split into fixed chunks;
-// each group sums the delta rows of every key segment of its chunk in
-// position order and adds the sum to its target; segments cut by a chunk
-// boundary leave partial sums that one owner combines in chunk order
-// (fix-up), and segments spanning many chunks (hot keys) are combined by
-// several blocks (push_long).
+// App. B.1.2).  Sorted (key, position) pairs are split into fixed chunks,
+// a block's groups taking consecutive chunks of one span; each group sums
+// the delta rows of every key segment of its chunk in position order and
+// adds the sum to its target.  A segment cut by chunk boundaries leaves a
+// partial sum per chunk; the block adds those of segments inside its span
+// in chunk order and applies them, and the partial sums of segments that run
+// past a span are added in span order by push_combine.
 #include "internal.cuh"
 #include "rowgroup.cuh"
 #include "store_launch.cuh"
@@ -60,13 +61,33 @@ __device__ __forceinline__ void apply_sum(const Store& s, const int32_t* mapw, u
 // (keys and source positions) in shared memory; its groups own consecutive
 // chunks of it.  A segment cut by chunk boundaries leaves a partial sum per
 // chunk (a tail piece in the chunk it starts in, head pieces in the chunks
-// it continues into); push_fixup / push_long add the pieces up.
+// it continues into).
 constexpr int kPushSpan = 3072;
 // resident push_chunks blocks per SM (its launch bounds)
 constexpr int push_blocks_per_sm(int C) { return C >= 4 ? 2 : 3; }
-// a segment cut by chunk boundaries and spanning at most this many further
-// chunks is combined by one group; longer ones (hot keys) by a whole block
-constexpr int kShortSpan = 8;
+
+// Sum of the pieces ph[m0 .. m1] (rows of D4 float4, lane's columns), added
+// in order to `tot`; loads issued in batches.
+template <int G, int C>
+__device__ __forceinline__ void add_pieces(const float4* ph4, uint64_t m0, uint64_t m1, uint32_t D4, int lane,
+                                           float4 (&tot)[C]) {
+  constexpr int UB = 8 / C > 0 ? 8 / C : 1;
+  for (uint64_t m = m0; m <= m1; m += UB) {
+    float4 t[UB][C];
+#pragma unroll
+    for (int u = 0; u < UB; ++u)
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        t[u][c] = (m + u <= m1 && col < D4) ? __ldcg(ph4 + (m + u) * D4 + col) : f4zero();
+      }
+#pragma unroll
+    for (int u = 0; u < UB; ++u)
+      if (m + u <= m1)
+#pragma unroll
+        for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+  }
+}
 
 template <int G, int C, int R>
 __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_kernel(Store s, PushArgs a0) {
@@ -92,6 +113,7 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
   float4* main4 = reinterpret_cast<float4*>(s.main);
   float4* ph4 = reinterpret_cast<float4*>(a.part_head);
   float4* pt4 = reinterpret_cast<float4*>(a.part_tail);
+  float4* sp4 = reinterpret_cast<float4*>(a.span_parts);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   uint32_t heads = 0;
   for (uint64_t P0 = (uint64_t)blockIdx.x * span; P0 < a.n; P0 += (uint64_t)gridDim.x * span) {
@@ -137,24 +159,34 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
     float4 run[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) run[c] = f4zero();
-    for (uint32_t p = p0; p < p1; p += R) {
-      // one round of loads: the delta rows
-      uint8_t f[R];
-      int32_t sl[R];
-      uint32_t k[R];
-      float4 d[R][C];
+    // software-pipelined: the delta rows of the next round are in flight
+    // while this round's are summed and applied
+    auto fetch = [&](uint32_t p, uint8_t (&f)[R], float4 (&d)[R][C]) {
 #pragma unroll
       for (int r = 0; r < R; ++r) {
         const bool v = p + r < p1;
         f[r] = v ? sf[p + r] : 0;
-        sl[r] = (f[r] & 7) == 7 ? ss[p + r] : -2;
-        k[r] = v ? sk[1 + p + r] : kNoKey;
         const uint32_t src = v ? sp[p + r] : 0u;
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
           d[r][c] = ((f[r] & 16) && col < D4) ? __ldg(d4 + (uint64_t)src * D4 + col) : f4zero();
         }
+      }
+    };
+    uint8_t f[R];
+    float4 d[R][C];
+    fetch(p0, f, d);
+    for (uint32_t p = p0; p < p1; p += R) {
+      uint8_t fn[R];
+      float4 dn[R][C];
+      fetch(p + R, fn, dn);
+      int32_t sl[R];
+      uint32_t k[R];
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        sl[r] = (f[r] & 7) == 7 ? ss[p + r] : -2;
+        k[r] = p + r < p1 ? sk[1 + p + r] : kNoKey;
       }
       // running sums in position order
 #pragma unroll
@@ -195,6 +227,77 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
           }
         }
       }
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        f[r] = fn[r];
+#pragma unroll
+        for (int c = 0; c < C; ++c) d[r][c] = dn[r][c];
+      }
+    }
+    // Pieces of the span's cut segments are in global memory (L2), visible
+    // to the whole block after the barrier.  A segment that begins in chunk
+    // gi and continues is combined here by group gi (its tail piece, then the
+    // head pieces of the chunks it covers, in chunk order) and applied when it
+    // ends inside the span; one that runs past the span leaves that sum as
+    // the span's tail piece, and the rows the span's first segment holds when
+    // it continues from the previous span are its head piece (group 0);
+    // push_combine adds span pieces up.
+    __syncthreads();
+    const uint32_t nch = (len + CH - 1) / CH;          // chunks of this span that hold rows
+    const uint64_t sidx = P0 / span;
+    auto chunk_end = [&](uint32_t m) { return (m + 1) * CH < len ? (m + 1) * CH : len; };
+    // last chunk m >= g the segment of key kk covers, given it reaches chunk g;
+    // out: it continues past the span
+    auto walk = [&](uint32_t g, uint32_t kk, bool& out) {
+      while (true) {
+        const uint32_t e = chunk_end(g);
+        const bool through = sk[e] == kk && sk[1 + e] == kk;   // last row kk, next row kk
+        if (!through || g + 1 >= nch) {
+          out = through;
+          return g;
+        }
+        ++g;
+      }
+    };
+    if (gi < (int)nch) {
+      const uint32_t kl = sk[p1];        // the chunk's last row
+      if (kl != kNoKey && sk[1 + p1] == kl) {
+        const bool whole = sk[1 + p0] == kl;
+        const bool began = !whole || P0 + p0 == 0 || sk[p0] != kl;
+        if (began) {
+          bool out = true;
+          const uint32_t g1 = (uint32_t)gi + 1 < nch ? walk(gi + 1, kl, out) : (uint32_t)gi;
+          float4 tot[C];
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            tot[c] = col < D4 ? __ldcg(pt4 + j * D4 + col) : f4zero();
+          }
+          if (g1 > (uint32_t)gi) add_pieces<G, C>(ph4, j + 1, P0 / CH + g1, D4, lane, tot);
+          if (out) {
+#pragma unroll
+            for (int c = 0; c < C; ++c) {
+              const uint32_t col = lane + c * G;
+              if (col < D4) sp4[(2 * sidx + 1) * D4 + col] = tot[c];
+            }
+          } else {
+            apply_sum<C>(s, mapw, kl, tot, lane, G);
+          }
+        }
+      }
+    }
+    if (gi == 0 && P0 > 0 && sk[1] != kNoKey && sk[0] == sk[1]) {
+      bool out = false;
+      const uint32_t g1 = walk(0, sk[1], out);
+      float4 tot[C];
+#pragma unroll
+      for (int c = 0; c < C; ++c) tot[c] = f4zero();
+      add_pieces<G, C>(ph4, P0 / CH, P0 / CH + g1, D4, lane, tot);
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const uint32_t col = lane + c * G;
+        if (col < D4) sp4[2 * sidx * D4 + col] = tot[c];
+      }
     }
   }
   uint32_t unused = 0;
@@ -205,242 +308,66 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
   }
 }
 
-// A segment that starts in chunk j and continues past it is owned by j: its
-// sum is j's tail piece plus the head pieces of chunks j+1 .. m_end.  Spans
-// of at most kShortSpan further chunks are combined here (loads issued
-// together); longer ones are listed for push_long_kernel.
+// Segments that run past a span: the span where one begins owns it; its sum
+// is that span's tail piece plus the head pieces of the spans it continues
+// into (found by a binary search for the last span whose first row holds
+// the key).  The groups of the block take those head pieces in strides, in
+// increasing order, then group 0 adds the tail piece and the group sums in
+// group order: a fixed order, whatever the number of spans.
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads) push_fixup_kernel(Store s, PushArgs a0, uint32_t* long_list,
-                                                              uint32_t* long_count) {
+__global__ void __launch_bounds__(kThreads) push_combine_kernel(Store s, PushArgs a0, uint64_t span,
+                                                                uint64_t nspans) {
   if (sort_failed(s.st)) return;
   const PushArgs a = resolve(a0);
-  const uint64_t CH = a.chunk;
+  constexpr int NG = kThreads / G;
+  __shared__ float4 part[NG][G * C];
   const int lane = threadIdx.x & (G - 1);
-  const uint64_t g = group_id<G>(), ng = group_count<G>();
+  const int gi = threadIdx.x / G;
   const uint32_t D4 = s.D >> 2;
-  const float4* ph4 = reinterpret_cast<const float4*>(a.part_head);
-  const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
+  const float4* sp4 = reinterpret_cast<const float4*>(a.span_parts);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
-  for (uint64_t j = g; j < a.nchunks; j += ng) {
-    const uint64_t p0 = j * CH;
-    const uint64_t p1 = p0 + CH;
-    if (p1 >= a.n) continue;
-    const uint32_t kl = a.skeys[p1 - 1];
-    if (kl == kNoKey || a.skeys[p1] != kl) continue;
-    if (p0 > 0 && a.skeys[p0 - 1] == kl) continue;           // started in an earlier chunk
-    bool cont[kShortSpan];   // cont[t]: the segment continues past chunk j+1+t
-#pragma unroll
-    for (int t = 0; t < kShortSpan; ++t) {
-      const uint64_t e = (j + 2 + t) * CH;
-      cont[t] = e < a.n && a.skeys[e] == kl;
+  for (uint64_t b = blockIdx.x; b < nspans; b += gridDim.x) {   // block-uniform
+    const uint64_t st = b * span;
+    const uint64_t en = st + span < a.n ? st + span : a.n;
+    const uint32_t kl = a.skeys[en - 1];
+    if (en >= a.n || kl == kNoKey || a.skeys[en] != kl) continue;
+    if (st > 0 && a.skeys[st - 1] == kl) continue;             // it began in an earlier span
+    uint64_t lo = b + 1, hi = nspans - 1;                      // last span whose first row holds kl
+    while (lo < hi) {
+      const uint64_t mid = (lo + hi + 1) / 2;
+      if (a.skeys[mid * span] == kl) lo = mid; else hi = mid - 1;
     }
-    int span = 0;            // further chunks after j+1 that the segment reaches
+    float4 acc[C];
 #pragma unroll
-    for (int t = 0; t < kShortSpan; ++t)
-      if (span == t && cont[t]) ++span;
-    if (span == kShortSpan) {
-      if (lane == 0) {
-        // last piece m whose first position still holds kl (a monotone predicate)
-        uint64_t lo = j + 1 + kShortSpan, hi = a.nchunks - 1;
-        while (lo < hi) {
-          const uint64_t mid = (lo + hi + 1) / 2;
-          if (a.skeys[mid * CH] == kl) lo = mid; else hi = mid - 1;
-        }
-        const uint32_t e = atomicAdd(long_count, 1u);
-        long_list[4 * e] = (uint32_t)j;
-        long_list[4 * e + 1] = (uint32_t)lo;
-        long_list[4 * e + 2] = 0;             // finished work items of this entry
-      }
-      continue;
-    }
-    float4 tot[C];
-#pragma unroll
-    for (int c = 0; c < C; ++c) {
-      const uint32_t col = lane + c * G;
-      tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
-    }
-    constexpr int UB = 8 / C > 0 ? 8 / C : 1;    // head pieces loaded together
-    for (int u0 = 0; u0 <= span; u0 += UB) {
+    for (int c = 0; c < C; ++c) acc[c] = f4zero();
+    constexpr int UB = 4 / C > 0 ? 4 / C : 1;
+    for (uint64_t m0 = b + 1 + gi; m0 <= lo; m0 += (uint64_t)NG * UB) {
       float4 t[UB][C];
 #pragma unroll
       for (int u = 0; u < UB; ++u)
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          t[u][c] = (u0 + u <= span && col < D4) ? ph4[(j + 1 + u0 + u) * D4 + col] : f4zero();
+          const uint64_t m = m0 + (uint64_t)u * NG;
+          t[u][c] = (m <= lo && col < D4) ? __ldcg(sp4 + 2 * m * D4 + col) : f4zero();
         }
 #pragma unroll
       for (int u = 0; u < UB; ++u)
-        if (u0 + u <= span)
 #pragma unroll
-          for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
+        for (int c = 0; c < C; ++c) acc[c] = f4add(acc[c], t[u][c]);
     }
-    apply_sum<C>(s, mapw, kl, tot, lane, G);
-  }
-}
-
-// Hot keys: a segment whose pieces run over more than kShortSpan further
-// chunks.  Its head pieces j+1 .. m_end are cut into work items of kLongSub
-// pieces, spread over all blocks; a block sums its item (groups take strided
-// pieces in increasing order, then the group sums in group order) into
-// long_parts.  The block that finishes an entry's last item sums the item
-// sums the same way (groups take strided items, then group order), adds the
-// tail piece and applies the total.  Every sum has a fixed order, so the
-// result does not depend on which block finishes last.
-constexpr uint32_t kLongSub = 32;
-constexpr uint32_t kLongSmem = 1024;   // long-list entries whose item bases sit in shared memory
-
-template <int G, int C>
-__global__ void __launch_bounds__(kThreads) push_long_kernel(Store s, PushArgs a0, uint32_t* long_list,
-                                                             const uint32_t* long_count) {
-  if (sort_failed(s.st)) return;
-  const PushArgs a = resolve(a0);
-  constexpr int NG = kThreads / G;
-  const uint64_t CH = a.chunk;
-  __shared__ float4 part[NG][G * C];
-  __shared__ int s_last;
-  const int lane = threadIdx.x & (G - 1);
-  const int gi = threadIdx.x / G;
-  const uint32_t D4 = s.D >> 2;
-  const float4* ph4 = reinterpret_cast<const float4*>(a.part_head);
-  const float4* pt4 = reinterpret_cast<const float4*>(a.part_tail);
-  float4* lp4 = reinterpret_cast<float4*>(a.long_parts);
-  const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
-  const uint32_t nl = *long_count;
-  // item bases of the first kLongSmem entries (block scan of their item
-  // counts), so that locating an item is a binary search in shared memory
-  __shared__ uint32_t s_base[kLongSmem + 1];
-  __shared__ uint32_t s_scan[kThreads / 32];
-  const uint32_t ns_tab = nl < kLongSmem ? nl : kLongSmem;
-  {
-    uint32_t carry = 0;
-    for (uint32_t e0 = 0; e0 < ns_tab; e0 += kThreads) {   // block-uniform trip count
-      const uint32_t e = e0 + threadIdx.x;
-      const uint32_t cnt = e < ns_tab ? (long_list[4 * e + 1] - long_list[4 * e] + kLongSub - 1) / kLongSub : 0u;
-      uint32_t x = cnt;
-      const int ln = threadIdx.x & 31, wp = threadIdx.x >> 5;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-        if (ln >= o) x += y;
-      }
-      if (ln == 31) s_scan[wp] = x;
-      __syncthreads();
-      uint32_t before = 0, total = 0;
-      for (int w2 = 0; w2 < kThreads / 32; ++w2) {
-        if (w2 < wp) before += s_scan[w2];
-        total += s_scan[w2];
-      }
-      if (e < ns_tab) s_base[e] = carry + before + x - cnt;
-      carry += total;
-      __syncthreads();
-    }
-    if (threadIdx.x == 0) s_base[ns_tab] = carry;
-    __syncthreads();
-  }
-  for (uint64_t q = blockIdx.x;; q += gridDim.x) {
-    // locate work item q: entry e, item it, first item of the entry `base`
-    uint64_t base = 0, it = 0, ns = 0, j = 0, m_end = 0;
-    uint32_t e = 0;
-    if (q < s_base[ns_tab]) {
-      uint32_t lo = 0, hi = ns_tab - 1;   // last entry whose base <= q
-      while (lo < hi) {
-        const uint32_t mid = (lo + hi + 1) / 2;
-        if (s_base[mid] <= q) lo = mid; else hi = mid - 1;
-      }
-      e = lo;
-      base = s_base[e];
-      j = long_list[4 * e];
-      m_end = long_list[4 * e + 1];
-      ns = (m_end - j + kLongSub - 1) / kLongSub;
-      it = q - base;
-    } else {
-      // entries past the table: walk them
-      base = s_base[ns_tab];
-      for (e = ns_tab; e < nl; ++e) {
-        j = long_list[4 * e];
-        m_end = long_list[4 * e + 1];
-        ns = (m_end - j + kLongSub - 1) / kLongSub;
-        if (q < base + ns) {
-          it = q - base;
-          break;
-        }
-        base += ns;
-      }
-      if (e == nl) break;
-    }
-    const uint64_t lo = j + 1 + it * kLongSub;
-    const uint64_t hi = lo + kLongSub - 1 < m_end ? lo + kLongSub - 1 : m_end;
-    float4 acc[C];
-#pragma unroll
-    for (int c = 0; c < C; ++c) acc[c] = f4zero();
-    constexpr int U = (kLongSub + NG - 1) / NG;
-    float4 t[U][C];
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        const uint64_t m = lo + gi + (uint64_t)u * NG;
-        t[u][c] = (m <= hi && col < D4) ? ph4[m * D4 + col] : f4zero();
-      }
-#pragma unroll
-    for (int u = 0; u < U; ++u)
-#pragma unroll
-      for (int c = 0; c < C; ++c) acc[c] = f4add(acc[c], t[u][c]);
 #pragma unroll
     for (int c = 0; c < C; ++c) part[gi][lane + c * G] = acc[c];
     __syncthreads();
     if (gi == 0) {
+      float4 tot[C];
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        float4 tot = f4zero();
-        for (int g2 = 0; g2 < NG; ++g2) tot = f4add(tot, part[g2][lane + c * G]);
-        if (col < D4) lp4[q * D4 + col] = tot;
+        tot[c] = col < D4 ? __ldcg(sp4 + (2 * b + 1) * D4 + col) : f4zero();
+        for (int g2 = 0; g2 < NG; ++g2) tot[c] = f4add(tot[c], part[g2][lane + c * G]);
       }
-    }
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) s_last = atomicAdd(long_list + 4 * e + 2, 1u) == (uint32_t)(ns - 1);
-    __syncthreads();
-    if (s_last) {   // block-uniform
-      // the entry's item sums: group g adds items g, g + NG, ... in order,
-      // then group 0 adds the tail piece and the group sums in group order
-      __threadfence();
-      float4 acc2[C];
-#pragma unroll
-      for (int c = 0; c < C; ++c) acc2[c] = f4zero();
-      constexpr int UB = 4 / C > 0 ? 4 / C : 1;
-      for (uint64_t i0 = gi; i0 < ns; i0 += (uint64_t)NG * UB) {
-        float4 t[UB][C];
-#pragma unroll
-        for (int u = 0; u < UB; ++u)
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + c * G;
-            const uint64_t it2 = i0 + (uint64_t)u * NG;
-            t[u][c] = (it2 < ns && col < D4) ? __ldcg(lp4 + (base + it2) * D4 + col) : f4zero();
-          }
-#pragma unroll
-        for (int u = 0; u < UB; ++u)
-#pragma unroll
-          for (int c = 0; c < C; ++c) acc2[c] = f4add(acc2[c], t[u][c]);
-      }
-#pragma unroll
-      for (int c = 0; c < C; ++c) part[gi][lane + c * G] = acc2[c];
-      __syncthreads();
-      if (gi == 0) {
-        const uint32_t kl = a.skeys[(j + 1) * CH - 1];
-        float4 tot[C];
-#pragma unroll
-        for (int c = 0; c < C; ++c) {
-          const uint32_t col = lane + c * G;
-          tot[c] = col < D4 ? pt4[j * D4 + col] : f4zero();
-          for (int g2 = 0; g2 < NG; ++g2) tot[c] = f4add(tot[c], part[g2][lane + c * G]);
-        }
-        apply_sum<C>(s, mapw, kl, tot, lane, G);
-      }
+      apply_sum<C>(s, mapw, kl, tot, lane, G);
     }
     __syncthreads();
   }
@@ -463,8 +390,7 @@ uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms) {
   return ch;
 }
 
-uint64_t push_long_list_words(uint64_t nchunks) { return 4 * (nchunks / 8 + 2) + 1; }
-uint64_t push_long_part_rows(uint64_t nchunks) { return nchunks / kLongSub + nchunks / 8 + 2; }
+uint64_t push_span_part_rows(uint64_t nchunks) { return 2 * (nchunks / 8 + 2); }
 
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream) {
   if (a.n == 0) return;
@@ -472,12 +398,14 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     constexpr int R = 4 / C > 0 ? 4 / C : 1;
     // one block per span: the block scheduler balances spans over the SMs
-    const uint64_t spans = (a.n + a.chunk * (kThreads / G) - 1) / (a.chunk * (kThreads / G));
-    note_launches(3);
+    const uint64_t span = a.chunk * (kThreads / G);
+    const uint64_t spans = (a.n + span - 1) / span;
+    note_launches(spans > 1 ? 2 : 1);
     push_chunks_kernel<G, C, R><<<(unsigned)spans, kThreads, 0, stream>>>(s, a);
-    push_fixup_kernel<G, C><<<grid_for(a.nchunks, G, sms), kThreads, 0, stream>>>(s, a, a.long_list,
-                                                                                 a.long_count);
-    push_long_kernel<G, C><<<(unsigned)sms * 2, kThreads, 0, stream>>>(s, a, a.long_list, a.long_count);
+    if (spans > 1) {
+      const unsigned grid = (unsigned)(spans < (uint64_t)sms * 8 ? spans : (uint64_t)sms * 8);
+      push_combine_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, a, span, spans);
+    }
   });
 }
 

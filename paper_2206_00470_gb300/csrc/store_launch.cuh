@@ -7,7 +7,9 @@ namespace adapm {
 
 // Arguments of the chunked push reduction.  skeys/spos: key-sorted keys and
 // their positions in `deltas` (n rows of D floats).  part_head / part_tail:
-// nchunks x D floats of scratch for segments cut by chunk boundaries.
+// nchunks x D floats of scratch for segments cut by chunk boundaries;
+// span_parts: push_span_part_rows(nchunks) x D floats for those cut by span
+// boundaries (a head and a tail row per span).
 struct PushArgs {
   const uint32_t* skeys;
   const uint32_t* spos;
@@ -18,9 +20,7 @@ struct PushArgs {
   uint64_t chunk;
   uint64_t nchunks;
   uint32_t worker;
-  uint32_t* long_list;    // push_long_list_words(nchunks) - 1 words of scratch
-  uint32_t* long_count;   // one word, zeroed by the caller
-  float* long_parts;      // push_long_part_rows(nchunks) x D floats of scratch
+  float* span_parts;
   // With plan_seq != 0, skeys / spos are a push plan and alt_keys / alt_pos
   // the sort made in its place; the kernels take the latter when
   // *plan_word == plan_seq (the plan did not match this push's keys).
@@ -30,9 +30,8 @@ struct PushArgs {
   uint32_t plan_seq = 0;
 };
 
-// Scratch sizes of the hot-key (long segment) combine for nchunks chunks.
-uint64_t push_long_list_words(uint64_t nchunks);
-uint64_t push_long_part_rows(uint64_t nchunks);
+// Rows of span_parts scratch for nchunks chunks (2 per span, spans of >= 8 chunks).
+uint64_t push_span_part_rows(uint64_t nchunks);
 
 // Rows per push chunk for value length D and a batch of n rows.
 uint64_t push_chunk_rows(uint32_t D, uint64_t n, int sms);
