@@ -2,12 +2,17 @@
 // the refcount events of advanceClock with the replicas they create and
 // destroy (Sec. 3, Sec. 4.1).
 //
-//   intent      the distinct keys of one call (hash set + stamps)       (Sec. 3)
-//   events      refcount +1 for every key of the opening intent lists,
-//               then -1 for the closing ones; transitions 0 -> 1 (create)
-//               and 1 -> 0 (evict)                                      (Sec. 3)
-//   evict       main += pending updates; free the slot                 (Sec. 4.1)
-//   create      val = main, pending = 0; take a slot                   (Sec. 4.1)
+//   intent        the distinct keys of one call (hash set + stamps)     (Sec. 3)
+//   events        refcount +1 for every key of the opening intent lists,
+//                 then -1 for the closing ones; transitions 0 -> 1
+//                 (create) and 1 -> 0 (evict); the last block of the
+//                 closing launch settles the advance's slot counts        (Sec. 3)
+//   evict_create  main += pending updates of every evicted replica, and
+//                 val = main, pending = 0 for every created one, the i-th
+//                 evicted slot going to the i-th created key             (Sec. 4.1)
+#include <utility>
+#include <vector>
+
 #include "internal.cuh"
 #include "rowgroup.cuh"
 #include "store_launch.cuh"
@@ -111,6 +116,36 @@ __device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32
   return eb.keys[l][i - pre[l]];
 }
 
+// Single thread, after every list append of the advance: the slot counts.
+// Evicted slots are handed to created keys pair by pair; only the surplus
+// of either list touches the free stack (pushes above the old top, or pops
+// from it).  The stack initially holds slots S-1 .. 0 (slot 0 on top) and
+// positions below S - high_water are never written, so popping down to
+// position p has used every slot below S - p.  Creations that need more
+// free slots than there are fail all together (ERR_NO_SLOTS).
+__device__ void settle_advance(DevState* st, int32_t S) {
+  const uint32_t ne = st->n_evict, nc = st->n_create;
+  const int32_t top = st->free_top;
+  uint32_t nc_ok = nc;
+  if (nc > ne && (int64_t)(nc - ne) > (int64_t)top) {
+    atomicOr(&st->errors, (uint32_t)ERR_NO_SLOTS);
+    nc_ok = 0;
+  }
+  st->adv_ne = ne;
+  st->adv_nc = nc_ok;
+  st->adv_top = top;
+  const int32_t ntop = top + (int32_t)ne - (int32_t)nc_ok;
+  st->free_top = ntop;
+  st->live += (int32_t)nc_ok - (int32_t)ne;
+  st->destroyed += ne;
+  st->created += nc_ok;
+  const int32_t lowest = ntop < top ? ntop : top;
+  if (S - lowest > st->high_water) st->high_water = S - lowest;
+  st->n_create = 0;   // ready for the next advance
+  st->n_evict = 0;
+  st->ev_done = 0;
+}
+
 // Refcount transitions of one advance of worker w.  All lists whose window
 // opens are applied first (START, rc += 1), then all lists whose window
 // closes (rc -= 1).  Every key of a closing list had a positive count before
@@ -134,7 +169,7 @@ __device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32
 // worker).  Four keys per thread and round; one list append per block and
 // round.  The order of a list is not specified.
 template <bool START>
-__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list) {
+__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list, int settle) {
   if (sort_failed(s.st)) return;
   constexpr int Q = 4;
   __shared__ uint32_t base_s;
@@ -250,161 +285,125 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
     }
     __syncthreads();
   }
+  if (!START && settle) {
+    // the last block to finish settles the advance's slot counts
+    __shared__ int last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      last = atomicAdd(&s.st->ev_done, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (last && threadIdx.x == 0) {
+      __threadfence();
+      settle_advance(s.st, (int32_t)s.S);
+    }
+  }
 }
 
-// evict: main[k] += acc[slot] for every listed slot (any worker's: a
-// relocation in this advance destroys another worker's replica); the freed
-// slot goes on the stack at free_top + i, so no list atomics are needed.  R
-// slots per row group at a time: the slots' owner records and pending rows
-// as one round of independent loads, together with the next round's slots.
+// evict_create: entry i of the advance evicts the i-th listed slot (any
+// worker's: a relocation destroys another worker's replica) -- main[k] +=
+// its pending row, by vector atomic adds since main[k] may receive two
+// pending rows in one advance (the leaving worker's and a relocated
+// holder's) -- and creates the i-th listed key of worker w, val = main,
+// pending = 0, in that same slot when there is one (the thread reads the
+// pending row before it overwrites it), else in a slot popped from the
+// stack; an evicted slot with no creation to take it is pushed.  A created
+// key is never one whose replica this advance destroys (a worker joins or
+// leaves a key, not both), so its main row is final.  R entries per row
+// group at a time; a round's loads (owner records, pending rows, main rows)
+// go out together with the next round's list entries.
 template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) evict_kernel(Store s,
-                                                                       const uint32_t* __restrict__ list) {
+__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(Store s, uint32_t w,
+                                                                              const uint32_t* __restrict__ evict_list,
+                                                                              const uint32_t* __restrict__ create_list) {
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
-  const uint32_t n = s.st->n_evict;
-  const int32_t top = s.st->free_top;
+  const uint32_t ne = s.st->adv_ne, nc = s.st->adv_nc;
+  const int32_t top = s.st->adv_top;
+  const uint64_t n = ne > nc ? ne : nc;
   float4* main4 = reinterpret_cast<float4*>(s.main);
-  const float4* acc4 = reinterpret_cast<const float4*>(s.acc);
-  const uint64_t g = group_id<G>(), ng = group_count<G>();
-  const uint64_t step = ng * R;
-  auto load_slots = [&](uint64_t i0, int32_t (&sl)[R]) {
-#pragma unroll
-    for (int r = 0; r < R; ++r) sl[r] = i0 + r < n ? (int32_t)list[i0 + r] : 0;
-  };
-  int32_t sl[R];
-  load_slots(g * R, sl);
-  for (uint64_t i0 = g * R; i0 < n; i0 += step) {
-    unsigned long long ow[R];
-    float4 ac[R][C];
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      ow[r] = i0 + r < n ? s.slot_owner[sl[r]] : 0ull;
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        ac[r][c] = (i0 + r < n && col < D4) ? acc4[(uint64_t)sl[r] * D4 + col] : f4zero();
-      }
-    }
-    int32_t sl1[R];
-    load_slots(i0 + step, sl1);
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      if (i0 + r >= n) break;
-      const uint32_t k = (uint32_t)ow[r], a = (uint32_t)(ow[r] >> 32);
-      // vector atomic adds: main[k] may receive two pending rows in one
-      // launch (the leaving worker's and a relocated holder's), and needs
-      // no load
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        if (col < D4) atomicAdd(main4 + (uint64_t)k * D4 + col, ac[r][c]);
-      }
-      if (lane == 0) {
-        if (s.dirty != nullptr) s.dirty[k] = 1;   // versioned refresh: main changed
-        // (always replicating, the events kernel that listed the slot has cleared its map entry)
-        if (s.own != nullptr) s.map[(uint64_t)a * s.K + k] = -1;
-        atomicAnd(s.holders + k, ~(1u << a));
-        s.slot_owner[sl[r]] = kEmptySlot;
-        s.free_stack[top + (int32_t)(i0 + r)] = sl[r];
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < R; ++r) sl[r] = sl1[r];
-  }
-}
-
-// Single thread: account the evictions, then reserve the creations.  The
-// stack initially holds slots S-1 .. 0 (slot 0 on top) and positions below
-// S - high_water are never written, so popping down to alloc_base has used
-// every slot below S - alloc_base.
-__global__ void alloc_kernel(DevState* st, int32_t S) {
-  const uint32_t ne = st->n_evict;
-  st->free_top += (int32_t)ne;
-  st->live -= (int32_t)ne;
-  st->destroyed += ne;
-  const uint32_t n = st->n_create;
-  if ((int64_t)n > (int64_t)st->free_top) {
-    st->errors |= ERR_NO_SLOTS;
-    st->n_create_ok = 0;
-    st->alloc_base = st->free_top;
-    return;
-  }
-  st->alloc_base = st->free_top - (int32_t)n;
-  st->free_top = st->alloc_base;
-  st->n_create_ok = n;
-  st->live += (int32_t)n;
-  st->created += n;
-  if (S - st->alloc_base > st->high_water) st->high_water = S - st->alloc_base;
-}
-
-// create: val = main[k], acc = 0, take a slot from the stack (R keys per
-// row group at a time, as in evict_kernel)
-template <int G, int C>
-__global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 4) create_kernel(Store s, uint32_t w,
-                                                                        const uint32_t* __restrict__ list) {
-  constexpr int R = 4 / C > 0 ? 4 / C : 1;
-  const int lane = threadIdx.x & (G - 1);
-  const uint32_t D4 = s.D >> 2;
-  const uint32_t n = s.st->n_create_ok;
-  const int32_t base = s.st->alloc_base;
-  int32_t* mapw = s.map + (uint64_t)w * s.K;
-  const float4* main4 = reinterpret_cast<const float4*>(s.main);
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
+  int32_t* mapw = s.map + (uint64_t)w * s.K;
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   const uint64_t step = ng * R;
-  // software-pipelined: a round loads the main rows of its keys and the list
-  // entries and slots of the next round together
-  auto load_entries = [&](uint64_t i0, uint32_t (&k)[R], int32_t (&sl)[R]) {
+  auto load_entries = [&](uint64_t i0, int32_t (&es)[R], uint32_t (&ck)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      const bool v = i0 + r < n;
-      k[r] = v ? list[i0 + r] : 0u;
-      // slots popped from the top of the stack: lowest free slots come first
-      sl[r] = v ? s.free_stack[base + (int32_t)(n - 1 - (i0 + r))] : 0;
+      const uint64_t i = i0 + r;
+      es[r] = i < ne ? (int32_t)evict_list[i] : -1;
+      ck[r] = i < nc ? create_list[i] : kNoKey;
     }
   };
-  uint32_t k[R];
-  int32_t sl[R];
-  load_entries(g * R, k, sl);
+  int32_t es[R];
+  uint32_t ck[R];
+  load_entries(g * R, es, ck);
   for (uint64_t i0 = g * R; i0 < n; i0 += step) {
-    float4 m[R][C];
-#pragma unroll
-    for (int r = 0; r < R; ++r)
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        m[r][c] = (i0 + r < n && col < D4) ? main4[(uint64_t)k[r] * D4 + col] : f4zero();
-      }
-    uint32_t k1[R];
-    int32_t sl1[R];
-    load_entries(i0 + step, k1, sl1);
+    int32_t cs[R];
+    unsigned long long ow[R];
+    float4 ac[R][C], mv[R][C];
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      if (i0 + r >= n) break;
+      const uint64_t i = i0 + r;
+      // slot of the creation: the paired evicted slot, else popped (top first)
+      cs[r] = ck[r] == kNoKey ? -1 : (es[r] >= 0 ? es[r] : s.free_stack[top - 1 - (int32_t)(i - ne)]);
+      ow[r] = es[r] >= 0 ? s.slot_owner[es[r]] : 0ull;
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
-        if (col < D4) {
-          val4[(uint64_t)sl[r] * D4 + col] = m[r][c];
-          acc4[(uint64_t)sl[r] * D4 + col] = f4zero();
+        ac[r][c] = (es[r] >= 0 && col < D4) ? acc4[(uint64_t)es[r] * D4 + col] : f4zero();
+        mv[r][c] = (ck[r] != kNoKey && col < D4) ? main4[(uint64_t)ck[r] * D4 + col] : f4zero();
+      }
+    }
+    int32_t es1[R];
+    uint32_t ck1[R];
+    load_entries(i0 + step, es1, ck1);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const uint64_t i = i0 + r;
+      if (es[r] >= 0) {
+        const uint32_t k = (uint32_t)ow[r], a = (uint32_t)(ow[r] >> 32);
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          if (col < D4) atomicAdd(main4 + (uint64_t)k * D4 + col, ac[r][c]);
+        }
+        if (lane == 0) {
+          if (s.dirty != nullptr) s.dirty[k] = 1;   // versioned refresh: main changed
+          // (always replicating, the events kernel that listed the slot has cleared its map entry)
+          if (s.own != nullptr) s.map[(uint64_t)a * s.K + k] = -1;
+          atomicAnd(s.holders + k, ~(1u << a));
+          if (ck[r] == kNoKey) {
+            s.slot_owner[es[r]] = kEmptySlot;
+            s.free_stack[top + (int32_t)(i - nc)] = es[r];
+          }
         }
       }
-      if (lane == 0) {
-        // versioned refresh: the new replica has seen every update (a stale
-        // replica of another worker is refreshed anyway: the key has two holders)
-        if (s.dirty != nullptr) s.dirty[k[r]] = 0;
-        mapw[k[r]] = sl[r];
-        atomicOr(s.holders + k[r], 1u << w);
-        s.slot_owner[sl[r]] = ((unsigned long long)w << 32) | k[r];
+      if (ck[r] != kNoKey) {
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          if (col < D4) {
+            val4[(uint64_t)cs[r] * D4 + col] = mv[r][c];
+            acc4[(uint64_t)cs[r] * D4 + col] = f4zero();
+          }
+        }
+        if (lane == 0) {
+          // versioned refresh: the new replica has seen every update (a stale
+          // replica of another worker is refreshed anyway: the key has two holders)
+          if (s.dirty != nullptr) s.dirty[ck[r]] = 0;
+          mapw[ck[r]] = cs[r];
+          atomicOr(s.holders + ck[r], 1u << w);
+          s.slot_owner[cs[r]] = ((unsigned long long)w << 32) | ck[r];
+        }
       }
     }
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      k[r] = k1[r];
-      sl[r] = sl1[r];
+      es[r] = es1[r];
+      ck[r] = ck1[r];
     }
   }
 }
@@ -422,34 +421,41 @@ void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint3
 
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
                    uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
-  // all opening lists first, then all closing lists, in batches of kEventLists
+  // all opening lists first, then all closing lists, in batches of kEventLists;
+  // the last closing launch (an empty one if no list closes) settles the slot counts
   const uint64_t cap_blocks = (uint64_t)sms * 8;
+  std::vector<std::pair<EventBatch, uint64_t>> batches[2];
   for (int pass = 0; pass < 2; ++pass) {
     const int sign = pass == 0 ? +1 : -1;
     EventBatch eb{};
     uint64_t cap = 0;
-    auto flush = [&]() {
-      if (eb.n == 0) return;
-      uint64_t b = (cap + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
-      if (b > cap_blocks) b = cap_blocks;
-      if (b == 0) b = 1;
-      note_launches(1);
-      if (pass == 0)
-        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list);
-      else
-        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, evict_list);
-      eb = EventBatch{};
-      cap = 0;
-    };
     for (int i = 0; i < nlists; ++i) {
       if (lists[i].sign != sign) continue;
       eb.keys[eb.n] = lists[i].keys;
       eb.count[eb.n] = lists[i].count;
       eb.n += 1;
       cap += lists[i].cap;   // the kernel covers the batch's lists as one index space
-      if (eb.n == kEventLists) flush();
+      if (eb.n == kEventLists) {
+        batches[pass].emplace_back(eb, cap);
+        eb = EventBatch{};
+        cap = 0;
+      }
     }
-    flush();
+    if (eb.n > 0 || (pass == 1 && batches[1].empty())) batches[pass].emplace_back(eb, cap);
+  }
+  for (int pass = 0; pass < 2; ++pass) {
+    for (size_t i = 0; i < batches[pass].size(); ++i) {
+      const EventBatch& eb = batches[pass][i].first;
+      uint64_t b = (batches[pass][i].second + 4 * kThreads - 1) / (4 * kThreads);   // 4 keys per thread
+      if (b > cap_blocks) b = cap_blocks;
+      if (b == 0) b = 1;
+      note_launches(1);
+      if (pass == 0)
+        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list, 0);
+      else
+        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, evict_list,
+                                                                    i + 1 == batches[1].size() ? 1 : 0);
+    }
   }
 }
 
@@ -458,12 +464,10 @@ void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list
                          cudaStream_t stream) {
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
-    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // list entries per group, as in the kernels
+    constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // list entries per group, as in the kernel
     const unsigned grid = grid_for((max_events + R - 1) / R, G, sms);
-    note_launches(3);
-    evict_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, evict_list);
-    alloc_kernel<<<1, 1, 0, stream>>>(s.st, (int32_t)s.S);
-    create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, create_list);
+    note_launches(1);
+    evict_create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list, create_list);
   });
 }
 

@@ -375,7 +375,7 @@ adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventLis
   const uint64_t max_events = ctx->s.own ? 2 * total : total;
   CK(pool_alloc(ctx, &create_list, total));
   CK(pool_alloc(ctx, &evict_list, max_events));
-  CK(cudaMemsetAsync(&ctx->dstate->n_create, 0, 2 * sizeof(uint32_t), ctx->stream));
+  // (the list counters are zero between advances: the last events launch clears them)
   launch_events(ctx->s, w, ev.data(), (int)ev.size(), create_list, evict_list, ctx->sms, ctx->stream);
   launch_evict_create(ctx->s, w, create_list, evict_list, max_events, ctx->sms, ctx->stream);
   pool_free(ctx, create_list);

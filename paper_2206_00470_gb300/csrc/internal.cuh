@@ -39,18 +39,18 @@ enum ErrBits : uint32_t {
 struct DevState {
   int32_t free_top;       // free slots on the stack
   int32_t high_water;     // slots [0, high_water) have been used
-  uint32_t n_create;      // keys appended to the create list of this advance
-  uint32_t n_evict;       // slots appended to the evict list of this advance
-  int32_t alloc_base;     // first stack index popped by this advance
-  uint32_t n_create_ok;   // creates that got a slot
+  uint32_t n_create;      // keys appended to the create list of this advance (0 between advances)
+  uint32_t n_evict;       // slots appended to the evict list of this advance (0 between advances)
+  int32_t adv_top;        // free_top before this advance's slots moved
+  uint32_t adv_nc;        // creations of this advance (0 if the slots ran out)
   uint32_t errors;        // ErrBits, sticky until read by adapm_wait
   uint32_t last_unique;   // distinct keys of the last push
   uint32_t plan_miss;     // sequence number of the last push whose plan did not match its keys
-  uint32_t pad0;
+  uint32_t adv_ne;        // evictions of this advance
   unsigned long long created;
   unsigned long long destroyed;
   int32_t live;
-  int32_t pad;
+  uint32_t ev_done;       // blocks of the closing events launch that finished (0 between advances)
   unsigned long long push_rows;       // rows pushed (cumulative)
   unsigned long long push_unique;     // distinct keys over all pushes (cumulative)
   unsigned long long sync_keys;       // keys merged by sync (cumulative)

@@ -57,10 +57,12 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
 // Refcount events of one advance of worker w: keys to create a replica of
 // for w go to create_list, replica slots to destroy (of w, and in relocation
 // mode of a worker the key is relocated to) to evict_list; the counters
-// n_create / n_evict in DevState must be zero.  With cap = the summed caps of
-// the lists, create_list needs cap entries and evict_list cap (always
-// replicate) or 2 * cap (relocation).  launch_evict_create applies both
-// lists; max_events bounds either list's length.
+// n_create / n_evict in DevState are zero between advances (the last events
+// launch settles the advance's slot counts and clears them).  With cap =
+// the summed caps of the lists, create_list needs cap entries and
+// evict_list cap (always replicate) or 2 * cap (relocation).
+// launch_evict_create applies both lists in one launch; max_events bounds
+// either list's length.
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
                    uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream);
 void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
