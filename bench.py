@@ -593,7 +593,8 @@ def manager_options(args):
     `config`."""
     return {"placement": "relocate" if args.relocate else "replicate", "action_timing": args.timing,
             "refresh": "versioned" if args.delta_refresh else "full",
-            "push_plans": not getattr(args, "no_push_plans", False)}
+            "push_plans": not getattr(args, "no_push_plans", False),
+            "pull": "bulk copies through shared memory" if getattr(args, "pull_staging", False) else "registers"}
 
 
 def run_ours(args, ws, rank, local, workload=None):
@@ -608,7 +609,8 @@ def run_ours(args, ws, rank, local, workload=None):
     init = wk.init_store()
     pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
                                 relocate=args.relocate, action_timing=args.timing,
-                                delta_refresh=args.delta_refresh, push_plans=not args.no_push_plans)
+                                delta_refresh=args.delta_refresh, push_plans=not args.no_push_plans,
+                                pull_staging=getattr(args, "pull_staging", False))
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -975,6 +977,8 @@ def main():
                     help="relocate a key to its only worker with active intent instead of always replicating")
     ap.add_argument("--delta-refresh", action="store_true",
                     help="versioned refresh: sync leaves a sole holder's value when nobody else wrote the key")
+    ap.add_argument("--pull-staging", action="store_true",
+                    help="pull rows through shared memory with bulk copies instead of through registers")
     ap.add_argument("--no-push-plans", action="store_true",
                     help="sort every push itself instead of using the sort made for its intent")
     ap.add_argument("--timing", default="start", choices=["start", "adaptive", "signal"],

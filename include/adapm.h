@@ -85,6 +85,10 @@ typedef struct {
   int32_t delta_refresh;     /* 0: sync refreshes every replica; 1: versioned refresh (see
                                 adapm_sync) */
   int32_t no_push_plans;     /* 0: push plans (see adapm_intent) are made and used; 1: never */
+  int32_t pull_staging;      /* adapm_pull moves rows 0: through registers (128-bit loads and
+                                streaming stores); 1: through shared memory by the bulk-copy
+                                engine (1-D cp.async.bulk per row, one bulk store per tile of
+                                output rows; used when out is 16-byte aligned) */
 } adapm_config;
 
 /* Action timing (Sec. 4.2).

@@ -46,6 +46,7 @@ class Config(ctypes.Structure):
         ("timing_lambda0", ctypes.c_double),
         ("delta_refresh", ctypes.c_int32),
         ("no_push_plans", ctypes.c_int32),
+        ("pull_staging", ctypes.c_int32),
     ]
 
 
@@ -202,11 +203,12 @@ class ParameterManager:
     delta_refresh   versioned refresh: sync leaves a sole holder's value when nobody else wrote the key
     push_plans      sort each intent's keys beside the library stream and let a push with the same keys
                     use that sort (adapm_intent); False sorts every push itself
+    pull_staging    pull rows through shared memory with bulk copies instead of through registers
     """
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
                  stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
-                 timing_lambda0=0.0, delta_refresh=False, push_plans=True):
+                 timing_lambda0=0.0, delta_refresh=False, push_plans=True, pull_staging=False):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -226,7 +228,7 @@ class ParameterManager:
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
                      ctypes.c_void_p(handle), int(self.relocate), ACTION_TIMING[action_timing],
                      float(timing_alpha), float(timing_p), float(timing_lambda0), int(bool(delta_refresh)),
-                     int(not push_plans))
+                     int(not push_plans), int(bool(pull_staging)))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:

@@ -15,7 +15,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libadapm.so")
-SOURCES = ["sort.cu", "store.cu", "push.cu", "advance.cu", "steps.cu", "capi.cu", "noalloc.cu"]
+SOURCES = ["sort.cu", "store.cu", "pull_bulk.cu", "push.cu", "advance.cu", "steps.cu", "capi.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC]
 

@@ -184,27 +184,34 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
   for (uint32_t b = blockIdx.x * blockDim.x * Q; b < n; b += stride) {   // block-uniform trip count
     uint32_t k[Q], old[Q], e0[Q], e1[Q];
     bool hit[Q], hit1[Q];
+    bool in[Q];   // a listed key in range (list entries are keys < K; anything else is skipped)
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
       const uint32_t i = b + q * blockDim.x + threadIdx.x;
       k[q] = i < n ? batch_key(eb, pre, i) : 0u;
+      in[q] = i < n && k[q] < s.K;
+      if (i < n && !in[q]) set_error(s.st, ERR_INTERNAL);
     }
+    // closing lists: the slot-map entry of every listed key is read with its
+    // atomic, not after it (only this thread touches it in this launch), so
+    // a transition costs one memory latency instead of two
+    int32_t msl[Q];
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
-      const uint32_t i = b + q * blockDim.x + threadIdx.x;
       old[q] = 1u;   // neither transition
-      if (i < n) old[q] = START ? atomicAdd(rcw + k[q], 1u) : atomicSub(rcw + k[q], 1u);
+      msl[q] = -1;
+      if (!START && in[q]) msl[q] = mapw[k[q]];
+      if (in[q]) old[q] = START ? atomicAdd(rcw + k[q], 1u) : atomicSub(rcw + k[q], 1u);
     }
 #pragma unroll
     for (int q = 0; q < Q; ++q) {
-      const uint32_t i = b + q * blockDim.x + threadIdx.x;
       hit1[q] = false;
       if (START) {
-        hit[q] = i < n && old[q] == 0u;
-        if (i < n && old[q] >= 65535u) set_error(s.st, ERR_REFCOUNT);
+        hit[q] = in[q] && old[q] == 0u;
+        if (in[q] && old[q] >= 65535u) set_error(s.st, ERR_REFCOUNT);
       } else {
-        hit[q] = i < n && old[q] == 1u;
-        if (i < n && old[q] == 0u) {   // more closings than openings: undo, report
+        hit[q] = in[q] && old[q] == 1u;
+        if (in[q] && old[q] == 0u) {   // more closings than openings: undo, report
           atomicAdd(rcw + k[q], 1u);
           set_error(s.st, ERR_REFCOUNT);
         }
@@ -238,7 +245,7 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
       uint32_t o[Q] = {}, hm[Q] = {};
 #pragma unroll
       for (int q = 0; q < Q; ++q) {
-        sl[q] = hit[q] ? mapw[k[q]] : -1;
+        sl[q] = hit[q] ? msl[q] : -1;
         if (reloc && hit[q]) {
           o[q] = s.own[k[q]];
           hm[q] = s.holders[k[q]];
@@ -329,12 +336,18 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(
   int32_t* mapw = s.map + (uint64_t)w * s.K;
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   const uint64_t step = ng * R;
+  // list entries out of range (slots >= S, keys >= K) are skipped and reported
   auto load_entries = [&](uint64_t i0, int32_t (&es)[R], uint32_t (&ck)[R]) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
       const uint64_t i = i0 + r;
-      es[r] = i < ne ? (int32_t)evict_list[i] : -1;
+      const uint32_t e = i < ne ? evict_list[i] : 0xFFFFFFFFu;
+      es[r] = e < s.S ? (int32_t)e : -1;
       ck[r] = i < nc ? create_list[i] : kNoKey;
+      if ((i < ne && e >= s.S) || (i < nc && ck[r] >= s.K)) {
+        set_error(s.st, ERR_INTERNAL);
+        if (ck[r] >= s.K) ck[r] = kNoKey;
+      }
     }
   };
   int32_t es[R];
@@ -350,6 +363,16 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(
       // slot of the creation: the paired evicted slot, else popped (top first)
       cs[r] = ck[r] == kNoKey ? -1 : (es[r] >= 0 ? es[r] : s.free_stack[top - 1 - (int32_t)(i - ne)]);
       ow[r] = es[r] >= 0 ? s.slot_owner[es[r]] : 0ull;
+      const bool bad_slot = ck[r] != kNoKey && (cs[r] < 0 || (uint64_t)cs[r] >= s.S);
+      const bool bad_owner = es[r] >= 0 && ((uint32_t)ow[r] >= s.K || (ow[r] >> 32) >= s.W);
+      if (bad_slot || bad_owner) {
+        set_error(s.st, ERR_INTERNAL);   // a free-stack entry or owner record out of range: skipped
+        if (bad_slot) {
+          cs[r] = -1;
+          ck[r] = kNoKey;
+        }
+        if (bad_owner) es[r] = -1;
+      }
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;

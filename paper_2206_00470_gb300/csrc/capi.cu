@@ -608,7 +608,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       cfg->action_timing < ADAPM_ACT_AT_START || cfg->action_timing > ADAPM_ACT_ON_SIGNAL ||
       !(cfg->timing_alpha >= 0.0 && cfg->timing_alpha <= 1.0) ||
       !(cfg->timing_p >= 0.0 && cfg->timing_p < 1.0) || !(cfg->timing_lambda0 >= 0.0) ||
-      (cfg->delta_refresh != 0 && cfg->delta_refresh != 1))
+      (cfg->delta_refresh != 0 && cfg->delta_refresh != 1) || (cfg->no_push_plans != 0 && cfg->no_push_plans != 1) ||
+      (cfg->pull_staging != 0 && cfg->pull_staging != 1))
     return ADAPM_EINVAL;
   adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
   if (!ctx) return ADAPM_ENOMEM;
@@ -836,7 +837,10 @@ adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
   CK(stage_out(ctx, out, n * ctx->s.D, &o));
   {
     ProfScope pk(ctx, 7);
-    launch_pull(ctx->s, (int)worker, in.dev, n, o.dev, ctx->sms, ctx->stream);
+    if (ctx->cfg.pull_staging && pull_bulk_fits(ctx->s.D, o.dev))
+      launch_pull_bulk(ctx->s, (int)worker, in.dev, n, o.dev, ctx->sms, ctx->stream);
+    else
+      launch_pull(ctx->s, (int)worker, in.dev, n, o.dev, ctx->sms, ctx->stream);
   }
   CK(finish_out(ctx, &o));
   pool_free(ctx, in.owned);
@@ -913,6 +917,8 @@ adapm_status adapm_wait(adapm_ctx* ctx) {
   if (errors & ERR_KEY_RANGE) return fail(ctx, ADAPM_ERANGE, "a key >= num_keys was passed");
   if (errors & ERR_NO_SLOTS) return fail(ctx, ADAPM_ENOMEM, "replica capacity exhausted");
   if (errors & ERR_REFCOUNT) return fail(ctx, ADAPM_ESTATE, "intent refcount overflow");
+  if (errors & ERR_INTERNAL)
+    return fail(ctx, ADAPM_ESTATE, "an index in the library's own state was out of range (element skipped)");
   return ADAPM_OK;
 }
 

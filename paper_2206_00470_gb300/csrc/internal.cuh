@@ -34,6 +34,8 @@ enum ErrBits : uint32_t {
   ERR_NO_SLOTS = 2u,    // replica capacity exhausted
   ERR_REFCOUNT = 4u,    // refcount over/underflow
   ERR_TIMEOUT = 8u,     // a bounded wait on another block gave up
+  ERR_INTERNAL = 16u,   // an index read from the library's own scratch or lists was out of
+                        // range: the element was skipped instead of accessed
 };
 
 struct DevState {

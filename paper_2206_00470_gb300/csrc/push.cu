@@ -133,7 +133,9 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
       const uint32_t k = sk[1 + i];
       uint8_t f = 0;
       int32_t slot = -2;
-      if (k != kNoKey) {
+      // (sorted keys are valid or the skip sentinel; anything else out of
+      // range, like a position outside the batch, is an internal error)
+      if (k < s.K && sp[i] < a.n) {
         const uint32_t cs = i - i % CH;                          // first row of the chunk
         const uint32_t ce = cs + CH < len ? cs + CH : len;        // end of the chunk
         const bool seg_begin = (P0 + i == 0) || sk[i] != k;       // sk[i] is the key of row i-1
@@ -149,6 +151,7 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
           if (slot < 0 && s.dirty != nullptr) s.dirty[k] = 1;
         }
       }
+      else if (k != kNoKey || sp[i] >= a.n) set_error(s.st, ERR_INTERNAL);
       sf[i] = f;
       ss[i] = slot;
     }
@@ -261,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
     };
     if (gi < (int)nch) {
       const uint32_t kl = sk[p1];        // the chunk's last row
-      if (kl != kNoKey && sk[1 + p1] == kl) {
+      if (kl < s.K && sk[1 + p1] == kl) {
         const bool whole = sk[1 + p0] == kl;
         const bool began = !whole || P0 + p0 == 0 || sk[p0] != kl;
         if (began) {
@@ -286,7 +289,7 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
         }
       }
     }
-    if (gi == 0 && P0 > 0 && sk[1] != kNoKey && sk[0] == sk[1]) {
+    if (gi == 0 && P0 > 0 && sk[1] < s.K && sk[0] == sk[1]) {
       bool out = false;
       const uint32_t g1 = walk(0, sk[1], out);
       float4 tot[C];
@@ -330,7 +333,7 @@ __global__ void __launch_bounds__(kThreads) push_combine_kernel(Store s, PushArg
     const uint64_t st = b * span;
     const uint64_t en = st + span < a.n ? st + span : a.n;
     const uint32_t kl = a.skeys[en - 1];
-    if (en >= a.n || kl == kNoKey || a.skeys[en] != kl) continue;
+    if (en >= a.n || kl >= s.K || a.skeys[en] != kl) continue;
     if (st > 0 && a.skeys[st - 1] == kl) continue;             // it began in an earlier span
     uint64_t lo = b + 1, hi = nspans - 1;                      // last span whose first row holds kl
     while (lo < hi) {

@@ -474,9 +474,15 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
           const uint32_t k = sm.sk[i];
           const uint32_t d = (k >> shift) & mask;
           const uint32_t pos = sm.base[d] + (i - sm.lofs[d]);
-          kout[pos] = k;
-          if (POS) vout[pos] = sm.sv[i];
-          if (more) tag = (((k >> nshift) & nmask) << 12) | (uint32_t)(pos / chunk);
+          // (positions come from the digit tables in scratch memory; one out of
+          // range is skipped and reported, never written)
+          if (pos < a.n) {
+            kout[pos] = k;
+            if (POS) vout[pos] = sm.sv[i];
+            if (more) tag = (((k >> nshift) & nmask) << 12) | (uint32_t)(pos / chunk);
+          } else {
+            set_error(a.st, ERR_INTERNAL);
+          }
         }
         if (more) {
           // one atomic per distinct (digit, chunk) of the warp

@@ -53,6 +53,11 @@ void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint3
                          uint32_t* count, int sms, cudaStream_t stream);
 void launch_pull(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
                  cudaStream_t stream);
+// The same pull with rows staged in shared memory by the bulk-copy engine
+// (pull_bulk.cu); usable when pull_bulk_fits(D, out): out 16-byte aligned.
+bool pull_bulk_fits(uint32_t D, const void* out);
+void launch_pull_bulk(const Store& s, int w, const uint32_t* keys, uint64_t n, float* out, int sms,
+                      cudaStream_t stream);
 void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream);
 // Refcount events of one advance of worker w: keys to create a replica of
 // for w go to create_list, replica slots to destroy (of w, and in relocation
