@@ -192,8 +192,8 @@ adapm_status adapm_push(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
  *     (ADAPM_EINVAL otherwise).
  *   - A push whose sort and partial-sum buffers exceed the 16 MiB returns
  *     ADAPM_EINVAL with the sizes in adapm_last_error().  On a 152-SM GPU
- *     every n up to about 420k rows fits at value_len 64, 510k at 200 and
- *     300, 280k at 512 and 14k at 1024.
+ *     every n up to about 790k rows fits at value_len 64, 800k at 200 and
+ *     300, 770k at 512 and 710k at 1024.
  *   - The first call on a device looks up the array's device address with
  *     cudaGetSymbolAddress; make that first call before any stream capture.
  *   - Every call (all contexts of the process) shares the one array: calls

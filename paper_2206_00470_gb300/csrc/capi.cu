@@ -420,9 +420,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   CK(pool_alloc(ctx, &hist, sort_scratch_words(n)));
   const uint64_t chunk = push_chunk_rows(ctx->s.D, n, ctx->sms);
   const uint64_t nchunks = (n + chunk - 1) / chunk;
-  float *ph = nullptr, *pt = nullptr, *sparts = nullptr;
-  CK(pool_alloc(ctx, &ph, nchunks * ctx->s.D));
-  CK(pool_alloc(ctx, &pt, nchunks * ctx->s.D));
+  float* sparts = nullptr;
   CK(pool_alloc(ctx, &sparts, push_span_part_rows(nchunks) * ctx->s.D));
   // the sort also clears the distinct-key counter
   uint32_t *sk = nullptr, *sp = nullptr;
@@ -430,7 +428,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
                &ctx->bar_base, &ctx->dstate->last_unique, nullptr, ctx->stream, &sk, &sp,
                plan ? &ctx->dstate->plan_miss : nullptr, seq));
   ctx->push_rows_host += n;
-  PushArgs a{sk, sp, n, drows, ph, pt, chunk, nchunks, w, sparts};
+  PushArgs a{sk, sp, n, drows, chunk, nchunks, w, sparts};
   if (plan) {
     a.skeys = plan->psk;
     a.spos = plan->psp;
@@ -445,8 +443,6 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   }
   for (uint32_t* p : {ka, kb, va, vb}) pool_free(ctx, p);
   pool_free(ctx, hist);
-  pool_free(ctx, ph);
-  pool_free(ctx, pt);
   pool_free(ctx, sparts);
   return check_launch(ctx, "push");
 }

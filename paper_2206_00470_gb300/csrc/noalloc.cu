@@ -59,7 +59,7 @@ bool is_device_ptr(const void* p) {
 
 // Byte offsets of the scratch regions of one push of n rows.
 struct Layout {
-  size_t ka, kb, va, vb, hist, ph, pt, sparts, total;
+  size_t ka, kb, va, vb, hist, sparts, total;
   uint64_t chunk, nchunks;
 };
 
@@ -78,8 +78,6 @@ Layout layout(uint32_t D, uint64_t n, int sms) {
   L.va = take(n * 4);
   L.vb = take(n * 4);
   L.hist = take(adapm::sort_scratch_words(n) * 4);
-  L.ph = take(L.nchunks * D * 4);
-  L.pt = take(L.nchunks * D * 4);
   L.sparts = take(adapm::push_span_part_rows(L.nchunks) * D * 4);
   L.total = off;
   return L;
@@ -147,8 +145,6 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
              sp,
              n,
              deltas,
-             reinterpret_cast<float*>(base + L.ph),
-             reinterpret_cast<float*>(base + L.pt),
              L.chunk,
              L.nchunks,
              worker,

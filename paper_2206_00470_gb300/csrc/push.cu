@@ -66,27 +66,12 @@ constexpr int kPushSpan = 3072;
 // resident push_chunks blocks per SM (its launch bounds)
 constexpr int push_blocks_per_sm(int C) { return C >= 4 ? 2 : 3; }
 
-// Sum of the pieces ph[m0 .. m1] (rows of D4 float4, lane's columns), added
-// in order to `tot`; loads issued in batches.
-template <int G, int C>
-__device__ __forceinline__ void add_pieces(const float4* ph4, uint64_t m0, uint64_t m1, uint32_t D4, int lane,
-                                           float4 (&tot)[C]) {
-  constexpr int UB = 8 / C > 0 ? 8 / C : 1;
-  for (uint64_t m = m0; m <= m1; m += UB) {
-    float4 t[UB][C];
-#pragma unroll
-    for (int u = 0; u < UB; ++u)
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        t[u][c] = (m + u <= m1 && col < D4) ? __ldcg(ph4 + (m + u) * D4 + col) : f4zero();
-      }
-#pragma unroll
-    for (int u = 0; u < UB; ++u)
-      if (m + u <= m1)
-#pragma unroll
-        for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], t[u][c]);
-  }
+// Dynamic shared memory of push_chunks: the head and tail piece of every
+// chunk (a row of G * C float4 per group each), then the staged span.
+template <int C>
+constexpr size_t push_chunks_smem() {
+  return 2 * (size_t)kThreads * C * sizeof(float4) + (kPushSpan + 2) * sizeof(uint32_t) +
+         kPushSpan * sizeof(uint32_t) + kPushSpan * sizeof(int32_t) + kPushSpan;
 }
 
 template <int G, int C, int R>
@@ -96,10 +81,13 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
   constexpr int NG = kThreads / G;
   const uint32_t CH = (uint32_t)a.chunk;            // rows per group, NG * CH <= kPushSpan
   const uint32_t span = NG * CH;
-  __shared__ uint32_t sk[kPushSpan + 2];   // sk[0]: key before the span; sk[1+len]: key after it
-  __shared__ uint32_t sp[kPushSpan];       // source row of each sorted position
-  __shared__ int32_t ss[kPushSpan];        // target slot of rows that end a whole segment
-  __shared__ uint8_t sf[kPushSpan];        // row flags (below)
+  extern __shared__ __align__(16) unsigned char dsm[];
+  float4* ph = reinterpret_cast<float4*>(dsm);                    // head piece of each chunk
+  float4* pt = ph + kThreads * C;                                 // tail piece of each chunk
+  uint32_t* sk = reinterpret_cast<uint32_t*>(pt + kThreads * C);  // sk[0]: key before the span; sk[1+len]: after it
+  uint32_t* sp = sk + kPushSpan + 2;                              // source row of each sorted position
+  int32_t* ss = reinterpret_cast<int32_t*>(sp + kPushSpan);       // target slot of rows that end a whole segment
+  uint8_t* sf = reinterpret_cast<uint8_t*>(ss + kPushSpan);       // row flags (below)
   // flags: bit0 a piece ends at this row, bit1 that piece began inside the
   // row's chunk, bit2 the key's segment ends here, bit3 a piece begins here,
   // bit4 the row holds a key (not a skipped one); a row with bits 0-2 all set
@@ -111,8 +99,6 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
   float4* val4 = reinterpret_cast<float4*>(s.val);
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   float4* main4 = reinterpret_cast<float4*>(s.main);
-  float4* ph4 = reinterpret_cast<float4*>(a.part_head);
-  float4* pt4 = reinterpret_cast<float4*>(a.part_tail);
   float4* sp4 = reinterpret_cast<float4*>(a.span_parts);
   const int32_t* mapw = s.map + (uint64_t)a.worker * s.K;
   uint32_t heads = 0;
@@ -158,7 +144,6 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
     __syncthreads();
     const uint32_t p0 = gi * CH;
     const uint32_t p1 = p0 + CH < len ? p0 + CH : len;
-    const uint64_t j = P0 / CH + gi;                 // global chunk index
     float4 run[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) run[c] = f4zero();
@@ -221,13 +206,11 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
             }
           }
         } else if (f[r] & 1) {
-          // a piece of a segment cut by a chunk boundary: partial sum
-          float4* dst = (f[r] & 2) ? pt4 : ph4;
+          // a piece of a segment cut by a chunk boundary: partial sum, kept
+          // in shared memory (a chunk has at most one head and one tail piece)
+          float4* dst = (f[r] & 2) ? pt : ph;
 #pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + c * G;
-            if (col < D4) dst[j * D4 + col] = d[r][c];
-          }
+          for (int c = 0; c < C; ++c) dst[gi * G * C + lane + c * G] = d[r][c];
         }
       }
 #pragma unroll
@@ -237,8 +220,8 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
         for (int c = 0; c < C; ++c) d[r][c] = dn[r][c];
       }
     }
-    // Pieces of the span's cut segments are in global memory (L2), visible
-    // to the whole block after the barrier.  A segment that begins in chunk
+    // Pieces of the span's cut segments are in shared memory, visible to the
+    // whole block after the barrier.  A segment that begins in chunk
     // gi and continues is combined here by group gi (its tail piece, then the
     // head pieces of the chunks it covers, in chunk order) and applied when it
     // ends inside the span; one that runs past the span leaves that sum as
@@ -272,11 +255,10 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
           const uint32_t g1 = (uint32_t)gi + 1 < nch ? walk(gi + 1, kl, out) : (uint32_t)gi;
           float4 tot[C];
 #pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + c * G;
-            tot[c] = col < D4 ? __ldcg(pt4 + j * D4 + col) : f4zero();
-          }
-          if (g1 > (uint32_t)gi) add_pieces<G, C>(ph4, j + 1, P0 / CH + g1, D4, lane, tot);
+          for (int c = 0; c < C; ++c) tot[c] = pt[gi * G * C + lane + c * G];
+          for (uint32_t m = gi + 1; m <= g1; ++m)
+#pragma unroll
+            for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], ph[m * G * C + lane + c * G]);
           if (out) {
 #pragma unroll
             for (int c = 0; c < C; ++c) {
@@ -294,8 +276,10 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
       const uint32_t g1 = walk(0, sk[1], out);
       float4 tot[C];
 #pragma unroll
-      for (int c = 0; c < C; ++c) tot[c] = f4zero();
-      add_pieces<G, C>(ph4, P0 / CH, P0 / CH + g1, D4, lane, tot);
+      for (int c = 0; c < C; ++c) tot[c] = ph[lane + c * G];
+      for (uint32_t m = 1; m <= g1; ++m)
+#pragma unroll
+        for (int c = 0; c < C; ++c) tot[c] = f4add(tot[c], ph[m * G * C + lane + c * G]);
 #pragma unroll
       for (int c = 0; c < C; ++c) {
         const uint32_t col = lane + c * G;
@@ -404,7 +388,16 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
     const uint64_t span = a.chunk * (kThreads / G);
     const uint64_t spans = (a.n + span - 1) / span;
     note_launches(spans > 1 ? 2 : 1);
-    push_chunks_kernel<G, C, R><<<(unsigned)spans, kThreads, 0, stream>>>(s, a);
+    constexpr size_t smem = push_chunks_smem<C>();
+    // the kernel's dynamic shared-memory limit is a per-device attribute
+    static bool attr_set[64] = {false};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+      cudaFuncSetAttribute(push_chunks_kernel<G, C, R>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (dev >= 0 && dev < 64) attr_set[dev] = true;
+    }
+    push_chunks_kernel<G, C, R><<<(unsigned)spans, kThreads, smem, stream>>>(s, a);
     if (spans > 1) {
       const unsigned grid = (unsigned)(spans < (uint64_t)sms * 8 ? spans : (uint64_t)sms * 8);
       push_combine_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, a, span, spans);

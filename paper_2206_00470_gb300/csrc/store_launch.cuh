@@ -6,17 +6,14 @@
 namespace adapm {
 
 // Arguments of the chunked push reduction.  skeys/spos: key-sorted keys and
-// their positions in `deltas` (n rows of D floats).  part_head / part_tail:
-// nchunks x D floats of scratch for segments cut by chunk boundaries;
-// span_parts: push_span_part_rows(nchunks) x D floats for those cut by span
-// boundaries (a head and a tail row per span).
+// their positions in `deltas` (n rows of D floats).  span_parts:
+// push_span_part_rows(nchunks) x D floats of scratch for the partial sums
+// of segments cut by span boundaries (a head and a tail row per span).
 struct PushArgs {
   const uint32_t* skeys;
   const uint32_t* spos;
   uint64_t n;
   const float* deltas;
-  float* part_head;
-  float* part_tail;
   uint64_t chunk;
   uint64_t nchunks;
   uint32_t worker;

@@ -93,14 +93,14 @@ def test_push_noalloc_dyadic_matches_oracle(gpu_lib):
 
 def test_push_noalloc_rejects_what_it_cannot_serve(gpu_lib):
     A = gpu_lib
-    K, D = 100, 1024
+    K, D = 100, 64
     pm = A.ParameterManager(K, D, 1)
     # host arrays would need staging buffers
     with pytest.raises(A.AdaPMError) as e:
         pm.push_noalloc(0, np.array([1, 2]), np.zeros((2, D), np.float32))
     assert e.value.status == A.EINVAL
-    # more rows than the 16 MiB scratch holds at value_len 1024
-    n = 40000
+    # more rows than the 16 MiB scratch holds (about 790k at value_len 64)
+    n = 900000
     with pytest.raises(A.AdaPMError) as e:
         pm.push_noalloc(0, torch.zeros(n, dtype=torch.int32, device="cuda"),
                         torch.zeros((n, D), device="cuda"))
