@@ -297,8 +297,7 @@ __global__ void __launch_bounds__(kThreads, push_blocks_per_sm(C)) push_chunks_k
 
 // Segments that run past a span: the span where one begins owns it; its sum
 // is that span's tail piece plus the head pieces of the spans it continues
-// into (found by a binary search for the last span whose first row holds
-// the key).  The groups of the block take those head pieces in strides, in
+// into (the spans whose first row holds the key, counted by the block).  The groups of the block take those head pieces in strides, in
 // increasing order, then group 0 adds the tail piece and the group sums in
 // group order: a fixed order, whatever the number of spans.
 template <int G, int C>
@@ -319,15 +318,20 @@ __global__ void __launch_bounds__(kThreads) push_combine_kernel(Store s, PushArg
     const uint32_t kl = a.skeys[en - 1];
     if (en >= a.n || kl >= s.K || a.skeys[en] != kl) continue;
     if (st > 0 && a.skeys[st - 1] == kl) continue;             // it began in an earlier span
-    uint64_t lo = b + 1, hi = nspans - 1;                      // last span whose first row holds kl
-    while (lo < hi) {
-      const uint64_t mid = (lo + hi + 1) / 2;
-      if (a.skeys[mid * span] == kl) lo = mid; else hi = mid - 1;
+    // the last span whose first row holds kl: the spans after b that do form
+    // a prefix (the keys are sorted), so the block tests kThreads of them at
+    // once and counts
+    uint64_t lo = b;
+    for (uint64_t m0 = b + 1; m0 < nspans; m0 += kThreads) {   // block-uniform
+      const uint64_t m = m0 + threadIdx.x;
+      const int cnt = __syncthreads_count(m < nspans && a.skeys[m * span] == kl);
+      lo += (uint64_t)cnt;
+      if (cnt < kThreads) break;
     }
     float4 acc[C];
 #pragma unroll
     for (int c = 0; c < C; ++c) acc[c] = f4zero();
-    constexpr int UB = 4 / C > 0 ? 4 / C : 1;
+    constexpr int UB = 8 / C > 0 ? 8 / C : 1;   // span pieces per group in flight
     for (uint64_t m0 = b + 1 + gi; m0 <= lo; m0 += (uint64_t)NG * UB) {
       float4 t[UB][C];
 #pragma unroll

@@ -260,19 +260,21 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     if (a.clear0) *a.clear0 = 0u;
     if (a.clear1) *a.clear1 = 0u;
   }
-  // an earlier sort gave up: the barrier state is unknown, so do nothing
-  if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
-  __syncthreads();
-  if (sm.abort) return;
-  // a verified plan already holds this sort's result: arrive at every barrier
-  // of the launch at once (the host counts them) and stop
-  if (a.plan_seq != 0u && ld_acquire(a.plan_word) != a.plan_seq) {
-    if (threadIdx.x == 0 && coop) {
+  // an earlier sort gave up (the barrier state is unknown): do nothing; a
+  // verified plan already holds this sort's result: arrive at every barrier
+  // of the launch at once (the host counts them) and stop.  Both words are
+  // read together by one thread.
+  if (threadIdx.x == 0) {
+    const uint32_t err = ld_acquire(&a.st->errors);
+    const uint32_t pw = a.plan_seq != 0u ? ld_acquire(a.plan_word) : 0u;
+    sm.abort = (err & ERR_TIMEOUT) ? 1 : ((a.plan_seq != 0u && pw != a.plan_seq) ? 2 : 0);
+    if (sm.abort == 2 && coop) {
       const unsigned long long nb = sort_barriers(a.passes);
       asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(&a.st->bar_arrivals), "l"(nb) : "memory");
     }
-    return;
   }
+  __syncthreads();
+  if (sm.abort) return;
   auto run = [&](int ph) { return coop || a.phase == ph; };
   uint32_t nbar = 0;
   const uint64_t chunk = (a.n + B - 1) / B;
@@ -662,12 +664,28 @@ __global__ void __launch_bounds__(kSortThreads) plan_verify_kernel(const uint32_
                                                                    uint64_t K, int allow_nokey, uint32_t seq,
                                                                    uint32_t* word, DevState* st) {
   bool bad = false, miss = false;
-  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (uint64_t)gridDim.x * blockDim.x) {
-    const uint32_t s = __ldg(sk + i);
-    const uint32_t pos = __ldg(sp + i);
-    const uint32_t k = pos < n ? __ldg(keys + pos) : s ^ 1u;
-    if (k >= K && !(allow_nokey && k == kNoKey)) bad = true;
-    miss |= s == kNoKey ? k < K : k != s;
+  constexpr int U = 4;   // positions per thread and round: their gathers go out together
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t i0 = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i0 < n; i0 += U * stride) {
+    uint32_t sv[U], pv[U], kv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t i = i0 + u * stride;
+      sv[u] = i < n ? __ldg(sk + i) : 0u;
+      pv[u] = i < n ? __ldg(sp + i) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t i = i0 + u * stride;
+      kv[u] = (i < n && pv[u] < n) ? __ldg(keys + pv[u]) : sv[u] ^ 1u;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (i0 + u * stride >= n) continue;
+      const uint32_t s = sv[u], k = kv[u];
+      if (k >= K && !(allow_nokey && k == kNoKey)) bad = true;
+      miss |= s == kNoKey ? k < K : k != s;
+    }
   }
   // the first warp to record this push's mismatch counts it
   if (__any_sync(0xFFFFFFFFu, miss) && (threadIdx.x & 31) == 0 && atomicExch(word, seq) != seq)
@@ -736,7 +754,7 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
 void launch_plan_verify(const uint32_t* keys, const uint32_t* sk, const uint32_t* sp, uint64_t n, uint64_t K,
                         bool allow_nokey, uint32_t seq, uint32_t* word, DevState* st, int sms, cudaStream_t stream) {
   if (n == 0) return;
-  uint64_t b = (n + kSortThreads * 4 - 1) / (kSortThreads * 4);
+  uint64_t b = (n + kSortThreads * 4 - 1) / (kSortThreads * 4);   // four positions per thread
   if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
   note_launches(1);
   plan_verify_kernel<<<(unsigned)b, kSortThreads, 0, stream>>>(keys, sk, sp, n, K, allow_nokey ? 1 : 0, seq, word,
