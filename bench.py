@@ -53,14 +53,14 @@ from synth import workloads as wl  # noqa: E402
 
 METRIC = "pulled+pushed keys/s and training samples/s on 1 GB300; % of HBM roofline"
 
-# DRAM bytes (read + write) of the push scatter kernels (push_chunks + push_fixup + push_long) per
-# pushed row, per workload, from the full ncu captures summarised in profiles/ (each on a smaller case
-# of the same workload, scaled by rows); a figure stands for the kernels only while their source is the
-# one captured (source_digest: first 16 hex digits of the sha256 of their code without comments), otherwise
-# the traffic is reported as null.
+# DRAM bytes (read + write) of the push scatter kernels (push_chunks + push_combine) per pushed row, per
+# workload, from the one-pass ncu captures summarised in profiles/ (each on a smaller case of the same
+# workload, scaled by rows); a figure stands for the kernels only while their source is the one captured
+# (source_digest: first 16 hex digits of the sha256 of their code without comments), otherwise the traffic
+# is reported as null.
 PUSH_SOURCES = ("paper_2206_00470_gb300/csrc/push.cu", "paper_2206_00470_gb300/csrc/rowgroup.cuh")
 PUSH_TRAFFIC = {
-    "mf": {"bytes_per_row": 83.35e6 / 65536, "sha256_16": "063dcdafb303627f"},   # profiles/push_scatter_mf_2Mx200K.md
+    "mf": {"bytes_per_row": 79.106e6 / 65536, "sha256_16": "b7ebddd50ef3a39f"},   # profiles/push_scatter_mf_2Mx200K.md
     "micro": {"bytes_per_row": None, "sha256_16": None},
 }
 
