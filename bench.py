@@ -585,7 +585,7 @@ def alg_bytes_per_step(wk, d, steps, relocate=False):
 
 
 COUNTERS = ("push_rows", "push_unique", "sync_keys", "sync_replicas", "sync_refreshed", "created", "destroyed",
-            "relocations", "planned_pushes", "plan_misses")
+            "relocations", "planned_pushes", "plan_misses", "early_advances", "early_undone")
 
 
 def manager_options(args):
@@ -594,6 +594,7 @@ def manager_options(args):
     return {"placement": "relocate" if args.relocate else "replicate", "action_timing": args.timing,
             "refresh": "versioned" if args.delta_refresh else "full",
             "push_plans": not getattr(args, "no_push_plans", False),
+            "early_events": not getattr(args, "no_early_events", False),
             "pull": "bulk copies through shared memory" if getattr(args, "pull_staging", False) else "registers"}
 
 
@@ -610,7 +611,8 @@ def run_ours(args, ws, rank, local, workload=None):
     pm = adapm.ParameterManager(wk.K, wk.D, wk.W, replica_capacity=wk.capacity, init_values=init,
                                 relocate=args.relocate, action_timing=args.timing,
                                 delta_refresh=args.delta_refresh, push_plans=not args.no_push_plans,
-                                pull_staging=getattr(args, "pull_staging", False))
+                                pull_staging=getattr(args, "pull_staging", False),
+                                early_events=not getattr(args, "no_early_events", False))
     del init
     torch.cuda.synchronize()
     setup_s = time.time() - t0
@@ -721,6 +723,7 @@ def run_ours(args, ws, rank, local, workload=None):
         "replica_events_per_step": {k: delta[k] / steps for k in ("created", "destroyed", "sync_replicas",
                                                                    "sync_refreshed", "sync_keys", "relocations")},
         "push_plans_per_step": {k: delta[k] / steps for k in ("planned_pushes", "plan_misses")},
+        "early_events_per_step": {k: delta[k] / steps for k in ("early_advances", "early_undone")},
         "setup_s": setup_s,
     }
     if e2e_ms is not None:
@@ -942,7 +945,7 @@ def run_reference(args, ws, rank):
 
 
 MICRO_KEYS = ("value", "unit", "ms_per_step", "config", "gpu_launches", "clocks", "roofline", "ops", "e2e",
-              "stats", "replica_events_per_step", "push_plans_per_step", "setup_s")
+              "stats", "replica_events_per_step", "push_plans_per_step", "early_events_per_step", "setup_s")
 
 
 def micro_args(args, zipf):
@@ -981,6 +984,8 @@ def main():
                     help="pull rows through shared memory with bulk copies instead of through registers")
     ap.add_argument("--no-push-plans", action="store_true",
                     help="sort every push itself instead of using the sort made for its intent")
+    ap.add_argument("--no-early-events", action="store_true",
+                    help="compute each advance's refcount events in the advance instead of beside the pull/push")
     ap.add_argument("--timing", default="start", choices=["start", "adaptive", "signal"],
                     help="act on an intent at its start clock, by Algorithm 1 at each sync, or when signalled")
     args = ap.parse_args()

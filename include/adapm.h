@@ -89,6 +89,9 @@ typedef struct {
                                 streaming stores); 1: through shared memory by the bulk-copy
                                 engine (1-D cp.async.bulk per row, one bulk store per tile of
                                 output rows; used when out is 16-byte aligned) */
+  int32_t no_early_events;   /* 0: a worker's next advance computes its refcount events early,
+                                beside the worker's pull and push (see adapm_advance_clock);
+                                1: never */
 } adapm_config;
 
 /* Action timing (Sec. 4.2).
@@ -162,7 +165,18 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
  * replicas for keys whose first intent became active are created (value
  * copied from main).  A key that stays active keeps its replica untouched.
  * With relocation, keys are relocated as the worker's intents start and end
- * (see adapm_create); this can destroy another worker's replica. */
+ * (see adapm_create); this can destroy another worker's replica.
+ *
+ * Early events (unless no_early_events; not with relocation or adaptive
+ * timing).  The refcount changes of the worker's next advance (which keys
+ * gain their first active intent, which lose their last) depend only on the
+ * worker's own intents.  So the worker's first adapm_pull, adapm_push or
+ * training step after an advance computes them for the intents recorded by
+ * then, on a stream of the library's own beside the library stream, and the
+ * advance only moves the rows.  If the advance's intents differ from those
+ * (one recorded or applied in between), the early changes are undone first.
+ * Results are the same either way; adapm_refcounts reports the counts of
+ * the worker's current clock.  adapm_wait also waits for that stream. */
 adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker);
 
 /* Read n rows: out[i] = worker's replica of keys[i] if it holds one, else the
@@ -302,6 +316,8 @@ typedef struct {
   uint64_t sync_refreshed;   /* replica values written by sync, cumulative */
   uint64_t planned_pushes;   /* pushes that checked a push plan (see adapm_intent), cumulative */
   uint64_t plan_misses;      /* of those, pushes whose keys differed, so they sorted, cumulative */
+  uint64_t early_advances;   /* advances whose refcount events ran early, cumulative */
+  uint64_t early_undone;     /* early events undone (the advance's intents changed), cumulative */
 } adapm_stats;
 
 adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out);

@@ -47,6 +47,7 @@ class Config(ctypes.Structure):
         ("delta_refresh", ctypes.c_int32),
         ("no_push_plans", ctypes.c_int32),
         ("pull_staging", ctypes.c_int32),
+        ("no_early_events", ctypes.c_int32),
     ]
 
 
@@ -69,6 +70,8 @@ class Stats(ctypes.Structure):
         ("sync_refreshed", ctypes.c_uint64),
         ("planned_pushes", ctypes.c_uint64),
         ("plan_misses", ctypes.c_uint64),
+        ("early_advances", ctypes.c_uint64),
+        ("early_undone", ctypes.c_uint64),
     ]
 
 
@@ -204,11 +207,14 @@ class ParameterManager:
     push_plans      sort each intent's keys beside the library stream and let a push with the same keys
                     use that sort (adapm_intent); False sorts every push itself
     pull_staging    pull rows through shared memory with bulk copies instead of through registers
+    early_events    compute the refcount changes of a worker's next advance beside its pull and push
+                    (adapm_advance_clock); False computes them in the advance
     """
 
     def __init__(self, num_keys, value_len, num_workers, replica_capacity=0, init_values=None,
                  stream=None, relocate=False, action_timing="start", timing_alpha=0.0, timing_p=0.0,
-                 timing_lambda0=0.0, delta_refresh=False, push_plans=True, pull_staging=False):
+                 timing_lambda0=0.0, delta_refresh=False, push_plans=True, pull_staging=False,
+                 early_events=True):
         self._lib = load()
         torch = _torch()
         if stream is None:
@@ -228,7 +234,7 @@ class ParameterManager:
         cfg = Config(self.K, self.D, self.W, int(replica_capacity), init.ptr,
                      ctypes.c_void_p(handle), int(self.relocate), ACTION_TIMING[action_timing],
                      float(timing_alpha), float(timing_p), float(timing_lambda0), int(bool(delta_refresh)),
-                     int(not push_plans), int(bool(pull_staging)))
+                     int(not push_plans), int(bool(pull_staging)), int(not early_events))
         h = ctypes.c_void_p()
         st = self._lib.adapm_create(ctypes.byref(cfg), ctypes.byref(h))
         if st != OK:

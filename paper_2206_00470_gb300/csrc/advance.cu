@@ -123,17 +123,15 @@ __device__ __forceinline__ uint32_t batch_key(const EventBatch& eb, const uint32
 // positions below S - high_water are never written, so popping down to
 // position p has used every slot below S - p.  Creations that need more
 // free slots than there are fail all together (ERR_NO_SLOTS).
-__device__ void settle_advance(DevState* st, int32_t S) {
-  const uint32_t ne = st->n_evict, nc = st->n_create;
-  const int32_t top = st->free_top;
-  uint32_t nc_ok = nc;
-  if (nc > ne && (int64_t)(nc - ne) > (int64_t)top) {
-    atomicOr(&st->errors, (uint32_t)ERR_NO_SLOTS);
-    nc_ok = 0;
-  }
-  st->adv_ne = ne;
-  st->adv_nc = nc_ok;
-  st->adv_top = top;
+__device__ __forceinline__ uint32_t creations_ok(uint32_t ne, uint32_t nc, int32_t top) {
+  return (nc > ne && (int64_t)(nc - ne) > (int64_t)top) ? 0u : nc;
+}
+
+// The free stack and the store's counters after an advance of ne evictions
+// and nc listed creations from stack top `top`; returns the creations made.
+__device__ uint32_t settle_counts(DevState* st, int32_t S, uint32_t ne, uint32_t nc, int32_t top) {
+  const uint32_t nc_ok = creations_ok(ne, nc, top);
+  if (nc_ok != nc) atomicOr(&st->errors, (uint32_t)ERR_NO_SLOTS);
   const int32_t ntop = top + (int32_t)ne - (int32_t)nc_ok;
   st->free_top = ntop;
   st->live += (int32_t)nc_ok - (int32_t)ne;
@@ -141,6 +139,15 @@ __device__ void settle_advance(DevState* st, int32_t S) {
   st->created += nc_ok;
   const int32_t lowest = ntop < top ? ntop : top;
   if (S - lowest > st->high_water) st->high_water = S - lowest;
+  return nc_ok;
+}
+
+__device__ void settle_advance(DevState* st, int32_t S) {
+  const uint32_t ne = st->n_evict, nc = st->n_create;
+  const int32_t top = st->free_top;
+  st->adv_ne = ne;
+  st->adv_nc = settle_counts(st, S, ne, nc, top);
+  st->adv_top = top;
   st->n_create = 0;   // ready for the next advance
   st->n_evict = 0;
   st->ev_done = 0;
@@ -168,15 +175,20 @@ __device__ void settle_advance(DevState* st, int32_t S) {
 // The create list takes keys (of worker w), the evict list slots (of any
 // worker).  Four keys per thread and round; one list append per block and
 // round.  The order of a list is not specified.
+//
+// Early events (AdvCounts given): the lists are computed ahead of the
+// advance, beside the worker's push, with their own counters; the map
+// entries stay until evict_create clears them, and evict_create settles.
 template <bool START>
-__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list, int settle) {
+__global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_list, int settle,
+                              AdvCounts* early) {
   if (sort_failed(s.st)) return;
   constexpr int Q = 4;
   __shared__ uint32_t base_s;
   uint32_t* rcw = s.rc + (uint64_t)w * s.K;
   int32_t* mapw_mut = s.map + (uint64_t)w * s.K;
   const int32_t* mapw = mapw_mut;
-  uint32_t* counter = START ? &s.st->n_create : &s.st->n_evict;
+  uint32_t* counter = early ? (START ? &early->nc : &early->ne) : (START ? &s.st->n_create : &s.st->n_evict);
   const bool reloc = s.own != nullptr;
   uint32_t pre[kEventLists + 1];
   const uint32_t n = batch_prefix(eb, pre);
@@ -272,7 +284,7 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
         // always replicating, the slot map entry is cleared here, where its line was just read
         // (nothing reads the map between this kernel and the eviction of the listed slot); with
         // relocation the eviction clears it, off this kernel's longer chain of dependent accesses
-        if (hit[q] && !reloc) mapw_mut[k[q]] = -1;
+        if (hit[q] && !reloc && !early) mapw_mut[k[q]] = -1;
       }
     }
     uint32_t c = 0, total, mtotal;
@@ -320,15 +332,31 @@ __global__ void events_kernel(Store s, uint32_t w, EventBatch eb, uint32_t* out_
 // leaves a key, not both), so its main row is final.  R entries per row
 // group at a time; a round's loads (owner records, pending rows, main rows)
 // go out together with the next round's list entries.
+//
+// After early events (AdvCounts given) every block takes the list lengths
+// from the counters and the stack top from the store (the same values in
+// every block: the store changes only after all blocks have finished),
+// evicted slots also clear their map entries, and the last block to finish
+// settles the advance.
 template <int G, int C>
 __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(Store s, uint32_t w,
                                                                               const uint32_t* __restrict__ evict_list,
-                                                                              const uint32_t* __restrict__ create_list) {
+                                                                              const uint32_t* __restrict__ create_list,
+                                                                              AdvCounts* early) {
   constexpr int R = 4 / C > 0 ? 4 / C : 1;
   const int lane = threadIdx.x & (G - 1);
   const uint32_t D4 = s.D >> 2;
-  const uint32_t ne = s.st->adv_ne, nc = s.st->adv_nc;
-  const int32_t top = s.st->adv_top;
+  uint32_t ne, nc;
+  int32_t top;
+  if (early) {
+    ne = early->ne;
+    top = s.st->free_top;
+    nc = creations_ok(ne, early->nc, top);
+  } else {
+    ne = s.st->adv_ne;
+    nc = s.st->adv_nc;
+    top = s.st->adv_top;
+  }
   const uint64_t n = ne > nc ? ne : nc;
   float4* main4 = reinterpret_cast<float4*>(s.main);
   float4* val4 = reinterpret_cast<float4*>(s.val);
@@ -395,8 +423,9 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(
         }
         if (lane == 0) {
           if (s.dirty != nullptr) s.dirty[k] = 1;   // versioned refresh: main changed
-          // (always replicating, the events kernel that listed the slot has cleared its map entry)
-          if (s.own != nullptr) s.map[(uint64_t)a * s.K + k] = -1;
+          // (always replicating, the events kernel that listed the slot has
+          // cleared its map entry, unless it ran early)
+          if (s.own != nullptr || early) s.map[(uint64_t)a * s.K + k] = -1;
           atomicAnd(s.holders + k, ~(1u << a));
           if (ck[r] == kNoKey) {
             s.slot_owner[es[r]] = kEmptySlot;
@@ -429,6 +458,39 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : 3) evict_create_kernel(
       ck[r] = ck1[r];
     }
   }
+  if (early) {
+    // the last block to finish settles the advance (all blocks have read
+    // the stack top by then) and clears the counters for the next one
+    __shared__ int last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      last = atomicAdd(&early->done, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (last && threadIdx.x == 0) {
+      __threadfence();
+      // (the counters and the stack top are unchanged since every block read them)
+      settle_counts(s.st, (int32_t)s.S, early->ne, early->nc, s.st->free_top);
+      early->nc = 0;
+      early->ne = 0;
+      early->done = 0;
+    }
+  }
+}
+
+// Undo early events whose advance did not happen as computed (a list was
+// added or applied after them): refcount -= 1 for every key of the opening
+// lists and += 1 for the closing ones, with no transitions (nothing else
+// touched the worker's counts or lists since).
+__global__ void events_undo_kernel(Store s, uint32_t w, EventBatch eb, int sign) {
+  uint32_t* rcw = s.rc + (uint64_t)w * s.K;
+  uint32_t pre[kEventLists + 1];
+  const uint32_t n = batch_prefix(eb, pre);
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+    const uint32_t k = batch_key(eb, pre, i);
+    if (k < s.K) atomicAdd(rcw + k, sign > 0 ? 0xFFFFFFFFu : 1u);
+  }
 }
 
 }  // namespace
@@ -442,12 +504,13 @@ void launch_intent_dedup(const Store& s, const uint32_t* keys, uint64_t n, uint3
   intent_dedup_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, keys, n, tag, out, count);
 }
 
-void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
-                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream) {
-  // all opening lists first, then all closing lists, in batches of kEventLists;
-  // the last closing launch (an empty one if no list closes) settles the slot counts
-  const uint64_t cap_blocks = (uint64_t)sms * 8;
-  std::vector<std::pair<EventBatch, uint64_t>> batches[2];
+namespace {
+
+// The opening (pass 0) and closing (pass 1) lists in batches of kEventLists,
+// each with its summed capacity; with `end` an empty closing batch stands in
+// when no list closes.
+void event_batches(const EventList* lists, int nlists, bool end,
+                   std::vector<std::pair<EventBatch, uint64_t>> (&batches)[2]) {
   for (int pass = 0; pass < 2; ++pass) {
     const int sign = pass == 0 ? +1 : -1;
     EventBatch eb{};
@@ -464,8 +527,20 @@ void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlist
         cap = 0;
       }
     }
-    if (eb.n > 0 || (pass == 1 && batches[1].empty())) batches[pass].emplace_back(eb, cap);
+    if (eb.n > 0 || (end && pass == 1 && batches[1].empty())) batches[pass].emplace_back(eb, cap);
   }
+}
+
+}  // namespace
+
+void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
+                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream,
+                   AdvCounts* early) {
+  // all opening lists first, then all closing lists; without `early` the
+  // last closing launch (an empty one if no list closes) settles the slot counts
+  const uint64_t cap_blocks = (uint64_t)sms * 8;
+  std::vector<std::pair<EventBatch, uint64_t>> batches[2];
+  event_batches(lists, nlists, early == nullptr, batches);
   for (int pass = 0; pass < 2; ++pass) {
     for (size_t i = 0; i < batches[pass].size(); ++i) {
       const EventBatch& eb = batches[pass][i].first;
@@ -474,23 +549,38 @@ void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlist
       if (b == 0) b = 1;
       note_launches(1);
       if (pass == 0)
-        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list, 0);
+        events_kernel<true><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, create_list, 0, early);
       else
-        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(s, w, eb, evict_list,
-                                                                    i + 1 == batches[1].size() ? 1 : 0);
+        events_kernel<false><<<(unsigned)b, kThreads, 0, stream>>>(
+            s, w, eb, evict_list, (!early && i + 1 == batches[1].size()) ? 1 : 0, early);
+    }
+  }
+}
+
+void launch_events_undo(const Store& s, uint32_t w, const EventList* lists, int nlists, int sms,
+                        cudaStream_t stream) {
+  std::vector<std::pair<EventBatch, uint64_t>> batches[2];
+  event_batches(lists, nlists, false, batches);
+  for (int pass = 0; pass < 2; ++pass) {
+    for (const auto& bc : batches[pass]) {
+      uint64_t b = (bc.second + kThreads - 1) / kThreads;
+      if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
+      if (b == 0) b = 1;
+      note_launches(1);
+      events_undo_kernel<<<(unsigned)b, kThreads, 0, stream>>>(s, w, bc.first, pass == 0 ? +1 : -1);
     }
   }
 }
 
 void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
                          const uint32_t* evict_list, uint64_t max_events, int sms,
-                         cudaStream_t stream) {
+                         cudaStream_t stream, AdvCounts* early) {
   dispatch_gc(s.D / 4, [&](auto Gc, auto Cc) {
     constexpr int G = decltype(Gc)::value, C = decltype(Cc)::value;
     constexpr uint64_t R = 4 / C > 0 ? 4 / C : 1;   // list entries per group, as in the kernel
     const unsigned grid = grid_for((max_events + R - 1) / R, G, sms);
     note_launches(1);
-    evict_create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list, create_list);
+    evict_create_kernel<G, C><<<grid, kThreads, 0, stream>>>(s, w, evict_list, create_list, early);
   });
 }
 

@@ -55,6 +55,18 @@ struct WorkerState {
   std::map<int64_t, std::vector<int64_t>> starts;   // clock -> lists whose window opens
   std::map<int64_t, std::vector<int64_t>> ends;     // clock -> lists whose window closes
   std::vector<int64_t> order;                       // recorded lists, oldest first
+  // Early events of the next advance (made at the worker's first push after
+  // its last advance): the lists they cover, the create and evict lists
+  // they fill, and the event after them on the early stream.
+  struct Early {
+    bool active = false;
+    int64_t clock = 0;                 // the clock the advance reaches
+    std::vector<int64_t> open, close;  // list ids, in advance order
+    uint32_t* create_list = nullptr;
+    uint32_t* evict_list = nullptr;
+    uint64_t cap = 0;
+    cudaEvent_t done = nullptr;
+  } early;
 };
 
 }  // namespace
@@ -104,6 +116,13 @@ struct adapm_ctx {
   std::vector<cudaEvent_t> spare_ready;
   uint32_t plan_seq = 0;
   uint64_t planned_pushes = 0;
+  // Early advance events run on early_stream, beside the library stream's
+  // push, with per-worker counters early_counts[w] (device, zero between
+  // advances).
+  cudaStream_t early_stream = nullptr;
+  AdvCounts* early_counts = nullptr;
+  uint64_t early_advances = 0;   // advances that used their early events
+  uint64_t early_undone = 0;     // early events taken back
 };
 
 namespace {
@@ -364,8 +383,120 @@ adapm_status check_ctx(adapm_ctx* ctx) {
 constexpr uint64_t kMaxN = 1ull << 31;
 
 // Refcount events of one worker -> destroy, then create replicas.
+// ---------------------------------------------------------------------------
+// Early advance events.  The refcount events of a worker's next advance
+// read and write only that worker's refcounts and read its slot map, which
+// nothing but its own advances changes (always replicating), so they can run
+// before the advance, beside the worker's pull and push: at the worker's
+// first pull, push or step after an advance, the lists whose window opens
+// or closes at its next clock are applied on early_stream, into lists and
+// counters of the worker's own.  The advance then waits for them and runs
+// evict_create alone, which clears the evicted map entries and settles.  If
+// the advance's lists are not the ones used (an intent recorded or applied
+// in between), the early events are undone and the advance runs in full.
+// Not with relocation (its events read other workers' state) or adaptive
+// timing (its openings happen at syncs).
+// ---------------------------------------------------------------------------
+bool early_enabled(const adapm_ctx* ctx) {
+  return !ctx->cfg.no_early_events && ctx->s.own == nullptr && ctx->cfg.action_timing != ADAPM_ACT_ADAPTIVE;
+}
+
+// The lists of worker w's advance to clock c: opening ones, closing ones.
+void advance_lists(const WorkerState& ws, int64_t c, std::vector<int64_t>& open, std::vector<int64_t>& close) {
+  open.clear();
+  close.clear();
+  auto it = ws.starts.find(c);
+  if (it != ws.starts.end()) open = it->second;
+  it = ws.ends.find(c);
+  if (it != ws.ends.end()) close = it->second;
+}
+
+std::vector<EventList> event_lists(adapm_ctx* ctx, const std::vector<int64_t>& open,
+                                   const std::vector<int64_t>& close) {
+  std::vector<EventList> ev;
+  for (int64_t id : open) {
+    const IntentList& L = ctx->lists[id];
+    ev.push_back(EventList{L.keys, L.count, L.cap, +1});
+  }
+  for (int64_t id : close) {
+    const IntentList& L = ctx->lists[id];
+    ev.push_back(EventList{L.keys, L.count, L.cap, -1});
+  }
+  return ev;
+}
+
+adapm_status early_make(adapm_ctx* ctx, uint32_t w) {
+  WorkerState& ws = ctx->workers[w];
+  if (!early_enabled(ctx) || ws.early.active) return ADAPM_OK;
+  WorkerState::Early E;
+  E.clock = ws.clock + 1;
+  advance_lists(ws, E.clock, E.open, E.close);
+  if (E.open.empty() && E.close.empty()) return ADAPM_OK;
+  if (!ctx->early_stream) CK(cudaStreamCreateWithFlags(&ctx->early_stream, cudaStreamNonBlocking));
+  const std::vector<EventList> ev = event_lists(ctx, E.open, E.close);
+  for (const auto& e : ev) E.cap += e.cap;
+  CK(pool_alloc(ctx, &E.create_list, E.cap));
+  CK(pool_alloc(ctx, &E.evict_list, E.cap));
+  cudaEvent_t after = nullptr;
+  CK(take_ready_event(ctx, &after));
+  CK(cudaEventRecord(after, ctx->stream));
+  CK(cudaStreamWaitEvent(ctx->early_stream, after, 0));
+  ctx->spare_ready.push_back(after);   // the wait has captured it
+  for (int64_t id : E.open)
+    if (ctx->lists[id].from_plan) CK(cudaStreamWaitEvent(ctx->early_stream, ctx->lists[id].ready, 0));
+  launch_events(ctx->s, w, ev.data(), (int)ev.size(), E.create_list, E.evict_list, ctx->sms, ctx->early_stream,
+                ctx->early_counts + w);
+  CK(take_ready_event(ctx, &E.done));
+  CK(cudaEventRecord(E.done, ctx->early_stream));
+  E.active = true;
+  ws.early = std::move(E);
+  return ADAPM_OK;
+}
+
+// The library stream waits for w's early events; their lists are freed
+// after what the stream does with them.
+adapm_status early_release(adapm_ctx* ctx, WorkerState::Early& E) {
+  CK(cudaStreamWaitEvent(ctx->stream, E.done, 0));
+  return ADAPM_OK;
+}
+
+void early_clear(adapm_ctx* ctx, WorkerState::Early& E) {
+  pool_free(ctx, E.create_list);
+  pool_free(ctx, E.evict_list);
+  ctx->spare_ready.push_back(E.done);
+  E = WorkerState::Early{};
+}
+
+adapm_status early_undo(adapm_ctx* ctx, uint32_t w) {
+  WorkerState::Early& E = ctx->workers[w].early;
+  if (!E.active) return ADAPM_OK;
+  adapm_status st = early_release(ctx, E);
+  if (st != ADAPM_OK) return st;
+  const std::vector<EventList> ev = event_lists(ctx, E.open, E.close);
+  launch_events_undo(ctx->s, w, ev.data(), (int)ev.size(), ctx->sms, ctx->stream);
+  CK(cudaMemsetAsync(ctx->early_counts + w, 0, sizeof(AdvCounts), ctx->stream));
+  early_clear(ctx, E);
+  ctx->early_undone += 1;
+  return check_launch(ctx, "early events (undo)");
+}
+
+adapm_status early_apply(adapm_ctx* ctx, uint32_t w) {
+  WorkerState::Early& E = ctx->workers[w].early;
+  adapm_status st = early_release(ctx, E);
+  if (st != ADAPM_OK) return st;
+  launch_evict_create(ctx->s, w, E.create_list, E.evict_list, E.cap, ctx->sms, ctx->stream,
+                      ctx->early_counts + w);
+  early_clear(ctx, E);
+  ctx->early_advances += 1;
+  return check_launch(ctx, "advance");
+}
+
 adapm_status apply_events(adapm_ctx* ctx, uint32_t w, const std::vector<EventList>& ev,
                           const std::vector<cudaEvent_t>& waits = {}) {
+  {
+    const adapm_status st = early_undo(ctx, w);   // the lists change: early events no longer hold
+    if (st != ADAPM_OK) return st;
+  }
   for (cudaEvent_t r : waits) CK(cudaStreamWaitEvent(ctx->stream, r, 0));
   uint64_t total = 0;
   for (const auto& e : ev) total += e.cap;
@@ -399,6 +530,10 @@ IntentList* find_plan(adapm_ctx* ctx, uint32_t w, uint64_t n) {
 adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint64_t n,
                          const float* drows, bool allow_nokey) {
   if (n == 0) return ADAPM_OK;
+  {
+    const adapm_status st = early_make(ctx, w);
+    if (st != ADAPM_OK) return st;
+  }
   uint32_t *ka = nullptr, *kb = nullptr, *va = nullptr, *vb = nullptr, *hist = nullptr;
   IntentList* plan = find_plan(ctx, w, n);
   uint32_t seq = 0;
@@ -605,7 +740,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       !(cfg->timing_alpha >= 0.0 && cfg->timing_alpha <= 1.0) ||
       !(cfg->timing_p >= 0.0 && cfg->timing_p < 1.0) || !(cfg->timing_lambda0 >= 0.0) ||
       (cfg->delta_refresh != 0 && cfg->delta_refresh != 1) || (cfg->no_push_plans != 0 && cfg->no_push_plans != 1) ||
-      (cfg->pull_staging != 0 && cfg->pull_staging != 1))
+      (cfg->pull_staging != 0 && cfg->pull_staging != 1) ||
+      (cfg->no_early_events != 0 && cfg->no_early_events != 1))
     return ADAPM_EINVAL;
   adapm_ctx* ctx = new (std::nothrow) adapm_ctx();
   if (!ctx) return ADAPM_ENOMEM;
@@ -651,7 +787,8 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
       !dmalloc((void**)&s.slot_owner, S * 8) || !dmalloc((void**)&s.free_stack, S * 4) ||
       !dmalloc((void**)&s.stamp, K * 4) || (cfg->relocate && !dmalloc((void**)&s.own, K * 2)) ||
       (cfg->delta_refresh && !dmalloc((void**)&s.dirty, K)) ||
-      !dmalloc((void**)&ctx->dstate, sizeof(DevState))) {
+      !dmalloc((void**)&ctx->dstate, sizeof(DevState)) ||
+      !dmalloc((void**)&ctx->early_counts, W * sizeof(AdvCounts))) {
     cudaGetLastError();
     return bail(ADAPM_ENOMEM);
   }
@@ -669,6 +806,7 @@ adapm_status adapm_create(const adapm_config* cfg, adapm_ctx** out) {
   ok &= cudaMemsetAsync(s.stamp, 0, K * 4, st) == cudaSuccess;   // intent tags start at 1
   if (s.own) ok &= cudaMemsetAsync(s.own, 0, K * 2, st) == cudaSuccess;   // home, no active worker
   if (s.dirty) ok &= cudaMemsetAsync(s.dirty, 0, K, st) == cudaSuccess;
+  ok &= cudaMemsetAsync(ctx->early_counts, 0, W * sizeof(AdvCounts), st) == cudaSuccess;
   DevState h{};
   h.free_top = (int32_t)S;
   ok &= cudaMemcpyAsync(ctx->dstate, &h, sizeof h, cudaMemcpyHostToDevice, st) == cudaSuccess;
@@ -686,6 +824,13 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   cudaSetDevice(ctx->device);
   if (ctx->stream) cudaStreamSynchronize(ctx->stream);
   if (ctx->plan_stream) cudaStreamSynchronize(ctx->plan_stream);
+  if (ctx->early_stream) cudaStreamSynchronize(ctx->early_stream);
+  for (auto& ws : ctx->workers) {
+    if (!ws.early.active) continue;
+    for (void* p : {(void*)ws.early.create_list, (void*)ws.early.evict_list})
+      if (p) cudaFree(p);
+    if (ws.early.done) cudaEventDestroy(ws.early.done);
+  }
   for (auto& kv : ctx->lists) {
     for (void* p : {(void*)kv.second.keys, (void*)kv.second.psk, (void*)kv.second.psp, kv.second.in_owned})
       if (p) cudaFree(p);
@@ -694,7 +839,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   for (auto e : ctx->spare_ready) cudaEventDestroy(e);
   Store& s = ctx->s;
   void* ptrs[] = {s.main, s.val, s.acc, s.map, s.rc, s.holders, s.slot_owner, s.free_stack,
-                  s.stamp, s.own, s.dirty, ctx->dstate};
+                  s.stamp, s.own, s.dirty, ctx->dstate, ctx->early_counts};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& t : ctx->pending) {
@@ -709,6 +854,7 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
   if (ctx->copy_in) cudaStreamDestroy(ctx->copy_in);
   if (ctx->stage_pool) cudaMemPoolDestroy(ctx->stage_pool);
   if (ctx->plan_stream) cudaStreamDestroy(ctx->plan_stream);
+  if (ctx->early_stream) cudaStreamDestroy(ctx->early_stream);
   if (ctx->plan_pool) cudaMemPoolDestroy(ctx->plan_pool);
   if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
   if (ctx->own_stream && ctx->stream) cudaStreamDestroy(ctx->stream);
@@ -791,6 +937,23 @@ adapm_status adapm_advance_clock(adapm_ctx* ctx, uint32_t worker) {
   WorkerState& ws = ctx->workers[worker];
   ws.clock += 1;
   const int64_t c = ws.clock;
+  if (ws.early.active) {
+    std::vector<int64_t> open, close;
+    advance_lists(ws, c, open, close);
+    if (ws.early.clock == c && open == ws.early.open && close == ws.early.close) {
+      // the events ran ahead: evict and create only
+      {
+        ProfScope ps(ctx, 1);
+        st = early_apply(ctx, worker);
+      }
+      ws.starts.erase(c);
+      ws.ends.erase(c);
+      for (int64_t id : close) CK(close_list(ctx, worker, id));
+      return st;
+    }
+    st = early_undo(ctx, worker);
+    if (st != ADAPM_OK) return st;
+  }
   std::vector<EventList> ev;
   std::vector<int64_t> closing;
   std::vector<cudaEvent_t> waits;   // plans that the opening lists' distinct keys come from
@@ -826,6 +989,8 @@ adapm_status adapm_pull(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, u
   if (worker >= ctx->s.W) return fail(ctx, ADAPM_EINVAL, "worker %u >= %u", worker, ctx->s.W);
   if (n > kMaxN || (n > 0 && (!keys || !out))) return fail(ctx, ADAPM_EINVAL, "bad pointers/n");
   if (n == 0) return ADAPM_OK;
+  st = early_make(ctx, worker);
+  if (st != ADAPM_OK) return st;
   ProfScope ps(ctx, 2);
   Input<uint32_t> in;
   CK(stage_in(ctx, keys, n, &in));
@@ -903,6 +1068,7 @@ adapm_status adapm_wait(adapm_ctx* ctx) {
   cudaSetDevice(ctx->device);
   CK(cudaStreamSynchronize(ctx->stream));
   if (ctx->plan_stream) CK(cudaStreamSynchronize(ctx->plan_stream));   // plans read the callers' keys
+  if (ctx->early_stream) CK(cudaStreamSynchronize(ctx->early_stream));
   uint32_t errors = 0;
   CK(cudaMemcpy(&errors, &ctx->dstate->errors, sizeof errors, cudaMemcpyDeviceToHost));
   if (errors) CK(cudaMemset(&ctx->dstate->errors, 0, sizeof errors));
@@ -948,6 +1114,8 @@ adapm_status adapm_mf_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* row_
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  st = early_make(ctx, worker);
+  if (st != ADAPM_OK) return st;
   {
     ProfScope ps(ctx, 5);
     launch_mf_step(ctx->s, worker, ir.dev, ic.dev, iv.dev, n, dim, adagrad != 0, lr, eps, o,
@@ -1001,6 +1169,8 @@ adapm_status adapm_complex_step(adapm_ctx* ctx, uint32_t worker, const uint32_t*
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  st = early_make(ctx, worker);
+  if (st != ADAPM_OK) return st;
   {
     ProfScope ps(ctx, 5);
     launch_complex_step(ctx->s, worker, ih.dev, ir.dev, it.dev, ineg.dev, n, n_neg, dim, lr, eps,
@@ -1051,6 +1221,8 @@ adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* ce
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
+  st = early_make(ctx, worker);
+  if (st != ADAPM_OK) return st;
   {
     ProfScope ps(ctx, 5);
     launch_sgns_step(ctx->s, worker, ic.dev, ix.dev, ineg.dev, n, n_ctx, n_neg, vocab, dim, lr, o,
@@ -1129,6 +1301,8 @@ adapm_status adapm_refcounts(adapm_ctx* ctx, uint32_t worker, const uint32_t* ke
   if (worker >= ctx->s.W || n > kMaxN || (n > 0 && (!keys || !out)))
     return fail(ctx, ADAPM_EINVAL, "bad arguments");
   if (n == 0) return ADAPM_OK;
+  st = early_undo(ctx, worker);   // the counts as of the worker's clock
+  if (st != ADAPM_OK) return st;
   Input<uint32_t> in;
   CK(stage_in(ctx, keys, n, &in));
   Output<uint32_t> o;
@@ -1193,6 +1367,8 @@ adapm_status adapm_get_stats(adapm_ctx* ctx, adapm_stats* out) {
   out->sync_refreshed = h.sync_refreshed;
   out->planned_pushes = ctx->planned_pushes;
   out->plan_misses = h.plan_misses;
+  out->early_advances = ctx->early_advances;
+  out->early_undone = ctx->early_undone;
   return ADAPM_OK;
 }
 

@@ -65,6 +65,16 @@ struct DevState {
   alignas(128) unsigned long long bar_arrivals;
 };
 
+// Counters of one worker's early advance events (computed ahead of the
+// advance, on a stream of their own): list lengths, and the blocks of the
+// evict_create launch that have finished.  Zero between advances.
+struct AdvCounts {
+  uint32_t nc;     // keys on the create list
+  uint32_t ne;     // slots on the evict list
+  uint32_t done;   // evict_create blocks finished
+  uint32_t pad;
+};
+
 // Plain view of the device state passed to kernels by value.
 struct Store {
   float* main;

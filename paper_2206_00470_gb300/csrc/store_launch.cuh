@@ -65,11 +65,20 @@ void launch_push(const Store& s, const PushArgs& a, int sms, cudaStream_t stream
 // evict_list cap (always replicate) or 2 * cap (relocation).
 // launch_evict_create applies both lists in one launch; max_events bounds
 // either list's length.
+// With `early` (always replicating only) the events run ahead of the
+// advance: the list lengths go to *early (zero before), the map entries of
+// the listed slots stay, nothing is settled; launch_evict_create with the
+// same `early` then clears those map entries and settles.  Early events
+// that are not followed by their advance are taken back by
+// launch_events_undo (refcounts only) on the same lists.
 void launch_events(const Store& s, uint32_t w, const EventList* lists, int nlists,
-                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream);
+                   uint32_t* create_list, uint32_t* evict_list, int sms, cudaStream_t stream,
+                   AdvCounts* early = nullptr);
+void launch_events_undo(const Store& s, uint32_t w, const EventList* lists, int nlists, int sms,
+                        cudaStream_t stream);
 void launch_evict_create(const Store& s, uint32_t w, const uint32_t* create_list,
                          const uint32_t* evict_list, uint64_t max_events, int sms,
-                         cudaStream_t stream);
+                         cudaStream_t stream, AdvCounts* early = nullptr);
 void launch_sync(const Store& s, uint64_t slot_bound, int sms, cudaStream_t stream);
 void launch_refcounts(const Store& s, uint32_t w, const uint32_t* keys, uint64_t n, uint32_t* out,
                       cudaStream_t stream);
