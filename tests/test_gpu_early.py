@@ -202,3 +202,27 @@ def test_relocation_and_adaptive_timing_never_run_early(gpu_lib, kw):
     st = pm.stats()
     assert st["early_advances"] == 0 and st["early_undone"] == 0
     pm.close()
+
+
+@pytest.mark.parametrize("host", ["pinned", "pageable"])
+def test_host_intent_keys_with_early_events(gpu_lib, host):
+    """Intents with host keys (staged copies) in the microbenchmark loop, early events on."""
+    K, D, W = 2500, 16, 2
+    init = dyadic_init(K, D, 17)
+    ops = loop_ops(29, K, D, W, 5, 600, 1, 2)
+    pm = gpu_lib.ParameterManager(K, D, W, init_values=torch.from_numpy(init).cuda())
+    ref = ParameterManagerOracle(K, D, W, init)
+    keep = []   # pinned inputs stay unchanged until adapm_wait; the staged device copies are the library's
+    for op in ops:
+        if op["op"] == "intent":
+            k = torch.from_numpy(np.asarray(op["keys"], dtype=np.int32))
+            if host == "pinned":
+                k = k.pin_memory()
+                keep.append(k)
+            pm.intent(op["w"], k, op["start"], op["end"])
+        else:
+            apply_gpu(pm, op)
+        apply_ref(ref, op)
+    assert pm.stats()["early_advances"] > 0
+    compare_full_state(pm, ref, K, W)
+    pm.close()
