@@ -247,7 +247,12 @@ __device__ __forceinline__ void load_rank(const SortArgs& a, const uint32_t* kin
 // Number of grid barriers one sort_kernel launch passes.
 __host__ __device__ constexpr uint32_t sort_barriers(int passes) { return 2u * (uint32_t)passes; }
 
-template <bool POS, int ITEMS>
+// What one sort launch runs: every phase with grid barriers between
+// (cooperative), or one phase of a phased sort.  A phased launch is compiled
+// with its own phase's code alone (registers, occupancy).
+enum SortKind { kSortAll = 0, kSortCount = 1, kSortScan = 2, kSortScatter = 3 };
+
+template <bool POS, int ITEMS, int KIND>
 __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   constexpr int SUB = kSortThreads * ITEMS;   // keys per sub-tile
   __shared__ SortSmem sm;
@@ -255,7 +260,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   const int warp = threadIdx.x >> 5;
   const uint32_t B = gridDim.x;
   const uint32_t b = blockIdx.x;
-  const bool coop = a.phase < 0;
+  constexpr bool coop = KIND == kSortAll;
   if (b == 0 && threadIdx.x == 0 && (coop || a.phase == 0)) {
     if (a.clear0) *a.clear0 = 0u;
     if (a.clear1) *a.clear1 = 0u;
@@ -276,6 +281,9 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   __syncthreads();
   if (sm.abort) return;
   auto run = [&](int ph) { return coop || a.phase == ph; };
+  constexpr bool has_count = KIND == kSortAll || KIND == kSortCount;
+  constexpr bool has_scan = KIND == kSortAll || KIND == kSortScan;
+  constexpr bool has_scatter = KIND == kSortAll || KIND == kSortScatter;
   uint32_t nbar = 0;
   const uint64_t chunk = (a.n + B - 1) / B;
   const uint64_t c0 = a.n < b * chunk ? a.n : b * chunk;
@@ -289,22 +297,34 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
   uint32_t* vout = a.va;
   uint32_t key[ITEMS], val[ITEMS], rank[ITEMS];
   bool bad = false;
-  // 0. first pass digit counts of the chunk (ranks kept when one sub-tile)
-  if (run(0)) {
+  // 0. first pass digit counts of the chunk (ranks kept when one sub-tile
+  // and the scatter follows in this launch)
+  if (has_count && run(0)) {
     const int nbits = a.per < a.bits ? a.per : a.bits;
     const uint32_t mask = (1u << nbits) - 1u;
-    if (single) {
+    if (single && coop) {
       load_rank<POS, ITEMS>(a, kin, vin, true, c0, c1, 0, nbits, key, val, rank, bad, sm);
     } else {
       for (int d = threadIdx.x; d < kDigits; d += kSortThreads) sm.cnt[d] = 0;
       __syncthreads();
-      for (uint64_t i = c0 + threadIdx.x; i < c1; i += kSortThreads) {
-        uint32_t k = __ldg(kin + i);
-        if (k >= a.K) {
-          if (!(a.allow_nokey && k == kNoKey)) bad = true;
-          k = kNoKey;
+      // ITEMS keys per thread and round, their loads issued together
+      for (uint64_t i0 = c0 + threadIdx.x; i0 < c1; i0 += (uint64_t)kSortThreads * ITEMS) {
+        uint32_t kk[ITEMS];
+#pragma unroll
+        for (int it = 0; it < ITEMS; ++it) {
+          const uint64_t i = i0 + (uint64_t)it * kSortThreads;
+          kk[it] = i < c1 ? __ldg(kin + i) : 0u;
         }
-        atomicAdd(&sm.cnt[k & mask], 1u);
+#pragma unroll
+        for (int it = 0; it < ITEMS; ++it) {
+          if (i0 + (uint64_t)it * kSortThreads >= c1) continue;
+          uint32_t k = kk[it];
+          if (k >= a.K) {
+            if (!(a.allow_nokey && k == kNoKey)) bad = true;
+            k = kNoKey;
+          }
+          atomicAdd(&sm.cnt[k & mask], 1u);
+        }
       }
       __syncthreads();
     }
@@ -329,7 +349,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     // round of coalesced loads, combined through shared memory; otherwise
     // one warp per digit row, read in batches.  Every block
     // also clears its own column of the next pass's table.
-    if (run(1 + 2 * p)) {
+    if (has_scan && run(1 + 2 * p)) {
     if (more)
       for (uint32_t d = threadIdx.x; d <= nmask; d += kSortThreads) tnext[(uint64_t)d * B + b] = 0u;
     if (B <= 16) {
@@ -420,7 +440,7 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     if (coop && !grid_barrier(a, nbar, sm)) return;
     // 2. scatter: digit bases, then the chunk's sub-tiles in order; each
     // written key is counted for the next pass in the chunk it lands in
-    if (run(2 + 2 * p)) {
+    if (has_scatter && run(2 + 2 * p)) {
     {
       uint32_t v[kDPT], local = 0;
 #pragma unroll
@@ -603,7 +623,7 @@ template <bool POS, int ITEMS>
 int sort_blocks_per_sm() {
   static const int occ = [] {
     int o = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS, ITEMS>, kSortThreads, 0) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, sort_kernel<POS, ITEMS, kSortAll>, kSortThreads, 0) !=
         cudaSuccess) {
       cudaGetLastError();
       o = 1;
@@ -626,7 +646,7 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   a.phase = -1;
   void* params[] = {&a};
   note_launches(1);
-  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, ITEMS>, dim3((unsigned)B),
+  const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, ITEMS, kSortAll>, dim3((unsigned)B),
                                                     dim3(kSortThreads), params, 0, stream);
   if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes) * B;
   return e;
@@ -647,7 +667,12 @@ cudaError_t launch_sort_phased(SortArgs& a, cudaStream_t stream) {
   note_launches((uint64_t)phases);
   for (int ph = 0; ph < phases; ++ph) {
     a.phase = ph;
-    sort_kernel<POS, ITEMS><<<(unsigned)B, kSortThreads, 0, stream>>>(a);
+    if (ph == 0)
+      sort_kernel<POS, ITEMS, kSortCount><<<(unsigned)B, kSortThreads, 0, stream>>>(a);
+    else if (ph & 1)
+      sort_kernel<POS, ITEMS, kSortScan><<<(unsigned)B, kSortThreads, 0, stream>>>(a);
+    else
+      sort_kernel<POS, ITEMS, kSortScatter><<<(unsigned)B, kSortThreads, 0, stream>>>(a);
   }
   return cudaGetLastError();
 }
