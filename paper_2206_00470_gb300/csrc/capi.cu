@@ -41,6 +41,7 @@ struct IntentList {
   // (and after the distinct keys, when they come from the plan: from_plan).
   uint32_t* psk = nullptr;
   uint32_t* psp = nullptr;
+  uint32_t* px = nullptr;     // the call's keys as given (what a matching push's keys equal)
   uint64_t n = 0;
   bool from_plan = false;
   cudaEvent_t ready = nullptr;
@@ -535,18 +536,17 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
     if (st != ADAPM_OK) return st;
   }
   uint32_t *ka = nullptr, *kb = nullptr, *va = nullptr, *vb = nullptr, *hist = nullptr;
+  // with a plan, the sort launch first checks on the device that the push's
+  // keys are the ones the plan was made from, and sorts (into this push's
+  // own arrays) only if they are not; the scatter kernels read the plan's
+  // arrays or the sort's by the same check
   IntentList* plan = find_plan(ctx, w, n);
   uint32_t seq = 0;
   if (plan) {
-    // check the plan on the device; the sort below runs only if it does not
-    // match (into this push's own arrays), and the scatter kernels read the
-    // plan's arrays or the sort's by the same check
     CK(cudaStreamWaitEvent(ctx->stream, plan->ready, 0));
     if (++ctx->plan_seq == 0) ctx->plan_seq = 1;
     seq = ctx->plan_seq;
     ctx->planned_pushes += 1;
-    launch_plan_verify(dkeys, plan->psk, plan->psp, n, ctx->s.K, allow_nokey, seq, &ctx->dstate->plan_miss,
-                       ctx->dstate, ctx->sms, ctx->stream);
   }
   CK(pool_alloc(ctx, &ka, n));
   CK(pool_alloc(ctx, &kb, n));
@@ -561,7 +561,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   uint32_t *sk = nullptr, *sp = nullptr;
   CK(sort_keys(dkeys, n, ctx->s.K, allow_nokey, ctx->bits, ka, kb, va, vb, hist, ctx->sms, ctx->dstate,
                &ctx->bar_base, &ctx->dstate->last_unique, nullptr, ctx->stream, &sk, &sp,
-               plan ? &ctx->dstate->plan_miss : nullptr, seq));
+               plan ? plan->px : nullptr, plan ? &ctx->dstate->plan_miss : nullptr, seq));
   ctx->push_rows_host += n;
   PushArgs a{sk, sp, n, drows, chunk, nchunks, w, sparts};
   if (plan) {
@@ -640,6 +640,7 @@ cudaError_t make_plan(adapm_ctx* ctx, IntentList& L, const uint32_t* keys, cudaE
   cudaStream_t ps = ctx->plan_stream;
   const uint64_t n = L.n;
   if ((e = cudaStreamWaitEvent(ps, after, 0)) != cudaSuccess) return e;
+  if ((e = cudaMemcpyAsync(L.px, keys, n * sizeof(uint32_t), cudaMemcpyDeviceToDevice, ps)) != cudaSuccess) return e;
   uint32_t *tk = nullptr, *tv = nullptr, *hist = nullptr, *tmp = nullptr;
   auto palloc = [&](uint32_t** p, size_t words) {
     return cudaMallocFromPoolAsync(reinterpret_cast<void**>(p), (words ? words : 1) * sizeof(uint32_t),
@@ -654,7 +655,7 @@ cudaError_t make_plan(adapm_ctx* ctx, IntentList& L, const uint32_t* keys, cudaE
   uint32_t *sk = nullptr, *sp = nullptr;
   e = sort_keys(keys, n, ctx->s.K, false, ctx->bits, odd ? L.psk : tk, odd ? tk : L.psk, odd ? L.psp : tv,
                 odd ? tv : L.psp, hist, ctx->sms, ctx->dstate, &no_barriers, nullptr, nullptr, ps, &sk, &sp,
-                nullptr, 0, /*phased=*/true);
+                nullptr, nullptr, 0, /*phased=*/true);
   if (e != cudaSuccess) return e;
   if (L.from_plan) compact_sorted_heads(L.psk, n, L.keys, L.count, tmp, ps);
   for (uint32_t* p : {tk, tv, hist, tmp}) cudaFreeAsync(p, ps);
@@ -672,7 +673,7 @@ cudaError_t close_list(adapm_ctx* ctx, uint32_t w, int64_t id) {
     e = cudaStreamWaitEvent(ctx->stream, L.ready, 0);
     ctx->spare_ready.push_back(L.ready);   // the wait has captured it; it can be recorded again
   }
-  for (void* p : {(void*)L.keys, (void*)L.psk, (void*)L.psp, L.in_owned}) pool_free(ctx, p);
+  for (void* p : {(void*)L.keys, (void*)L.psk, (void*)L.psp, (void*)L.px, L.in_owned}) pool_free(ctx, p);
   auto& order = ctx->workers[w].order;
   order.erase(std::remove(order.begin(), order.end(), id), order.end());
   ctx->lists.erase(id);
@@ -832,7 +833,8 @@ adapm_status adapm_destroy(adapm_ctx* ctx) {
     if (ws.early.done) cudaEventDestroy(ws.early.done);
   }
   for (auto& kv : ctx->lists) {
-    for (void* p : {(void*)kv.second.keys, (void*)kv.second.psk, (void*)kv.second.psp, kv.second.in_owned})
+    for (void* p : {(void*)kv.second.keys, (void*)kv.second.psk, (void*)kv.second.psp, (void*)kv.second.px,
+                    kv.second.in_owned})
       if (p) cudaFree(p);
     if (kv.second.ready) cudaEventDestroy(kv.second.ready);
   }
@@ -892,6 +894,7 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
     if (plan) {
       CK(pool_alloc(ctx, &L.psk, n));
       CK(pool_alloc(ctx, &L.psp, n));
+      CK(pool_alloc(ctx, &L.px, n));
     }
     // a window that opens two or more clocks ahead takes its distinct keys
     // from the plan; one that opens at the next advance (or is active now)
@@ -1111,6 +1114,8 @@ adapm_status adapm_mf_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* row_
   const uint64_t m = 2 * n;
   StepOut o{};
   o.loss_blocks = step_loss_blocks(ctx->sms);
+  o.loss_out = loss_out ? lo.dev : nullptr;   // summed by the step kernel's last block
+  o.loss_done = &ctx->dstate->loss_done;
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
@@ -1121,7 +1126,6 @@ adapm_status adapm_mf_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* row_
     launch_mf_step(ctx->s, worker, ir.dev, ic.dev, iv.dev, n, dim, adagrad != 0, lr, eps, o,
                    ctx->sms, ctx->stream);
   }
-  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
   {
     ProfScope ps(ctx, 3);
     st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
@@ -1166,6 +1170,8 @@ adapm_status adapm_complex_step(adapm_ctx* ctx, uint32_t worker, const uint32_t*
   const uint64_t m = n * (3 + (uint64_t)n_neg);
   StepOut o{};
   o.loss_blocks = step_loss_blocks(ctx->sms);
+  o.loss_out = loss_out ? lo.dev : nullptr;   // summed by the step kernel's last block
+  o.loss_done = &ctx->dstate->loss_done;
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
@@ -1176,7 +1182,6 @@ adapm_status adapm_complex_step(adapm_ctx* ctx, uint32_t worker, const uint32_t*
     launch_complex_step(ctx->s, worker, ih.dev, ir.dev, it.dev, ineg.dev, n, n_neg, dim, lr, eps,
                         o, ctx->sms, ctx->stream);
   }
-  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
   {
     ProfScope ps(ctx, 3);
     st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
@@ -1218,6 +1223,8 @@ adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* ce
   const uint64_t m = n * per;
   StepOut o{};
   o.loss_blocks = step_loss_blocks(ctx->sms);
+  o.loss_out = loss_out ? lo.dev : nullptr;   // summed by the step kernel's last block
+  o.loss_done = &ctx->dstate->loss_done;
   CK(pool_alloc(ctx, &o.dkeys, m));
   CK(pool_alloc(ctx, &o.drows, m * ctx->s.D));
   CK(pool_alloc(ctx, &o.loss_part, o.loss_blocks));
@@ -1228,7 +1235,6 @@ adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* ce
     launch_sgns_step(ctx->s, worker, ic.dev, ix.dev, ineg.dev, n, n_ctx, n_neg, vocab, dim, lr, o,
                      ctx->sms, ctx->stream);
   }
-  if (loss_out) launch_loss_reduce(o.loss_part, o.loss_blocks, lo.dev, ctx->stream);
   {
     ProfScope ps(ctx, 3);
     st = push_device(ctx, worker, o.dkeys, m, o.drows, true);

@@ -53,6 +53,7 @@ struct DevState {
   unsigned long long destroyed;
   int32_t live;
   uint32_t ev_done;       // blocks of the closing events launch that finished (0 between advances)
+  uint32_t loss_done;     // blocks of a training step that finished (0 between steps)
   unsigned long long push_rows;       // rows pushed (cumulative)
   unsigned long long push_unique;     // distinct keys over all pushes (cumulative)
   unsigned long long sync_keys;       // keys merged by sync (cumulative)
@@ -127,10 +128,14 @@ __device__ __forceinline__ bool sort_failed(const DevState* st) {
 // up, the kernel sets ERR_TIMEOUT and returns; every kernel that consumes a
 // sort checks that bit first and does nothing while it is set.
 //
-// Plans: with plan_word non-null the launch sorts only if *plan_word ==
-// plan_seq when it runs (plan_verify stored a mismatch); otherwise its
-// blocks account their grid barriers and return, leaving ka/kb/va/vb as
-// they are (the caller's verified plan holds the result).
+// Plans (cooperative launch only): with plan_keys and plan_word, the blocks
+// first compare raw with plan_keys, the keys a plan was sorted from,
+// position by position (out-of-range keys all counting as the sentinel); a
+// mismatch stores plan_seq in *plan_word and counts a plan miss.  After one
+// more grid barrier the launch sorts only if *plan_word == plan_seq;
+// otherwise its blocks account their remaining barriers and return, leaving
+// ka/kb/va/vb as they are (the plan holds the result).  Out-of-range keys
+// are reported by the check as the sort would.
 // phased = true runs the sort as 1 + 2 * passes ordinary launches (kernel
 // boundaries instead of grid barriers, *bar_base untouched): for a stream
 // that runs beside other work, where a cooperative launch would wait for
@@ -141,15 +146,8 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
                       DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
                       cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out,
-                      const uint32_t* plan_word = nullptr, uint32_t plan_seq = 0, bool phased = false);
-
-// Checks a plan (sk, sp: the stable key sort of an earlier key list) against
-// the n keys of a push: stores seq in *word unless keys[sp[i]] == sk[i] for
-// every i (out-of-range keys matching the sentinel); sets ERR_KEY_RANGE for
-// an out-of-range push key as the sort would.
-void launch_plan_verify(const uint32_t* keys, const uint32_t* sk, const uint32_t* sp, uint64_t n, uint64_t K,
-                        bool allow_nokey, uint32_t seq, uint32_t* word, DevState* st, int sms,
-                        cudaStream_t stream);
+                      const uint32_t* plan_keys = nullptr, uint32_t* plan_word = nullptr, uint32_t plan_seq = 0,
+                      bool phased = false);
 
 // The distinct valid keys of a sorted array, ascending, into out; count to *count.
 void compact_sorted_heads(const uint32_t* sk, uint64_t n, uint32_t* out, uint32_t* count, uint32_t* tmp,

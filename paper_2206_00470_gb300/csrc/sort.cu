@@ -130,7 +130,11 @@ struct SortArgs {
   uint32_t* clear0;              // words set to zero by the launch (nullptr: none)
   uint32_t* clear1;
   unsigned long long bar_base;   // st->bar_arrivals when the launch starts
-  const uint32_t* plan_word;     // with plan_seq != 0: the sort runs only if *plan_word == plan_seq
+  // Plan check (cooperative launch): with plan_keys, the blocks first compare
+  // raw with plan_keys position by position; a mismatch stores plan_seq in
+  // *plan_word, and after a grid barrier the sort runs only if it did.
+  const uint32_t* plan_keys;
+  uint32_t* plan_word;
   uint32_t plan_seq;
   int phase;                     // -1: every phase, grid barriers between (cooperative launch);
                                  // k >= 0: phase k alone (0 count, 1 + 2p scan, 2 + 2p scatter of pass p)
@@ -265,27 +269,56 @@ __global__ void __launch_bounds__(kSortThreads, 4) sort_kernel(SortArgs a) {
     if (a.clear0) *a.clear0 = 0u;
     if (a.clear1) *a.clear1 = 0u;
   }
-  // an earlier sort gave up (the barrier state is unknown): do nothing; a
-  // verified plan already holds this sort's result: arrive at every barrier
-  // of the launch at once (the host counts them) and stop.  Both words are
-  // read together by one thread.
-  if (threadIdx.x == 0) {
-    const uint32_t err = ld_acquire(&a.st->errors);
-    const uint32_t pw = a.plan_seq != 0u ? ld_acquire(a.plan_word) : 0u;
-    sm.abort = (err & ERR_TIMEOUT) ? 1 : ((a.plan_seq != 0u && pw != a.plan_seq) ? 2 : 0);
-    if (sm.abort == 2 && coop) {
-      const unsigned long long nb = sort_barriers(a.passes);
-      asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(&a.st->bar_arrivals), "l"(nb) : "memory");
-    }
-  }
+  // an earlier sort gave up (the barrier state is unknown): do nothing
+  if (threadIdx.x == 0) sm.abort = (ld_acquire(&a.st->errors) & ERR_TIMEOUT) ? 1 : 0;
   __syncthreads();
   if (sm.abort) return;
+  uint32_t nbar = 0;
+  if (coop && a.plan_keys) {
+    // the plan holds this sort's result iff the push's keys equal the keys it
+    // was made from at every position (out-of-range keys all counting as the
+    // sentinel); every key is read once, so out-of-range keys are reported
+    // here as the sort's first pass would
+    constexpr int U = 4;
+    bool miss = false, bad = false;
+    const uint64_t stride = (uint64_t)gridDim.x * kSortThreads;
+    for (uint64_t i0 = (uint64_t)b * kSortThreads + threadIdx.x; i0 < a.n; i0 += U * stride) {
+      uint32_t kv[U], xv[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const uint64_t i = i0 + u * stride;
+        kv[u] = i < a.n ? __ldg(a.raw + i) : 0u;
+        xv[u] = i < a.n ? __ldg(a.plan_keys + i) : 0u;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (i0 + u * stride >= a.n) continue;
+        const uint32_t k = kv[u], x = xv[u];
+        if (k >= a.K && !(a.allow_nokey && k == kNoKey)) bad = true;
+        miss |= (k < a.K ? k : kNoKey) != (x < a.K ? x : kNoKey);
+      }
+    }
+    if (__any_sync(0xFFFFFFFFu, miss) && lane == 0 && atomicExch(a.plan_word, a.plan_seq) != a.plan_seq)
+      atomicAdd(&a.st->plan_misses, 1ull);
+    if (__any_sync(0xFFFFFFFFu, bad) && lane == 0) set_error(a.st, ERR_KEY_RANGE);
+    if (!grid_barrier(a, nbar, sm)) return;
+    // the plan matched: arrive at every later barrier of the launch at once
+    // (the host counts them) and stop
+    if (threadIdx.x == 0) {
+      sm.abort = ld_acquire(a.plan_word) != a.plan_seq ? 2 : 0;
+      if (sm.abort == 2) {
+        const unsigned long long nb = sort_barriers(a.passes);
+        asm volatile("red.release.gpu.global.add.u64 [%0], %1;" ::"l"(&a.st->bar_arrivals), "l"(nb) : "memory");
+      }
+    }
+    __syncthreads();
+    if (sm.abort) return;
+  }
   auto run = [&](int ph) { return coop || a.phase == ph; };
   constexpr bool has_count = KIND == kSortAll || KIND == kSortCount;
   constexpr bool has_scan = KIND == kSortAll || KIND == kSortScan;
   constexpr bool has_scatter = KIND == kSortAll || KIND == kSortScatter;
-  uint32_t nbar = 0;
-  const uint64_t chunk = (a.n + B - 1) / B;
+    const uint64_t chunk = (a.n + B - 1) / B;
   const uint64_t c0 = a.n < b * chunk ? a.n : b * chunk;
   const uint64_t c1 = a.n < c0 + chunk ? a.n : c0 + chunk;
   const bool single = c1 - c0 <= (uint64_t)SUB;
@@ -648,7 +681,7 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   note_launches(1);
   const cudaError_t e = cudaLaunchCooperativeKernel((const void*)sort_kernel<POS, ITEMS, kSortAll>, dim3((unsigned)B),
                                                     dim3(kSortThreads), params, 0, stream);
-  if (e == cudaSuccess) *bar_base += (unsigned long long)sort_barriers(a.passes) * B;
+  if (e == cudaSuccess) *bar_base += (unsigned long long)(sort_barriers(a.passes) + (a.plan_keys ? 1u : 0u)) * B;
   return e;
 }
 
@@ -677,47 +710,6 @@ cudaError_t launch_sort_phased(SortArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-// Plan check of a push: for every sorted position i, the push's key at
-// position sp[i] must equal sk[i] (both out of range where sk[i] is the
-// sentinel).  Then (sk, sp) is exactly the stable key sort of the push's
-// keys, since sk is sorted and sp a permutation.  A mismatch anywhere
-// stores `seq` in *word.  Every push key is read once (sp is a
-// permutation), so out-of-range keys are reported here as the sort would.
-__global__ void __launch_bounds__(kSortThreads) plan_verify_kernel(const uint32_t* __restrict__ keys,
-                                                                   const uint32_t* __restrict__ sk,
-                                                                   const uint32_t* __restrict__ sp, uint64_t n,
-                                                                   uint64_t K, int allow_nokey, uint32_t seq,
-                                                                   uint32_t* word, DevState* st) {
-  bool bad = false, miss = false;
-  constexpr int U = 4;   // positions per thread and round: their gathers go out together
-  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
-  for (uint64_t i0 = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i0 < n; i0 += U * stride) {
-    uint32_t sv[U], pv[U], kv[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const uint64_t i = i0 + u * stride;
-      sv[u] = i < n ? __ldg(sk + i) : 0u;
-      pv[u] = i < n ? __ldg(sp + i) : 0u;
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const uint64_t i = i0 + u * stride;
-      kv[u] = (i < n && pv[u] < n) ? __ldg(keys + pv[u]) : sv[u] ^ 1u;
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (i0 + u * stride >= n) continue;
-      const uint32_t s = sv[u], k = kv[u];
-      if (k >= K && !(allow_nokey && k == kNoKey)) bad = true;
-      miss |= s == kNoKey ? k < K : k != s;
-    }
-  }
-  // the first warp to record this push's mismatch counts it
-  if (__any_sync(0xFFFFFFFFu, miss) && (threadIdx.x & 31) == 0 && atomicExch(word, seq) != seq)
-    atomicAdd(&st->plan_misses, 1ull);
-  if (__any_sync(0xFFFFFFFFu, bad) && (threadIdx.x & 31) == 0) set_error(st, ERR_KEY_RANGE);
-}
-
 }  // namespace
 
 int bits_for(uint64_t num_keys) {
@@ -738,15 +730,16 @@ int sort_passes(int bits) { return plan_for(bits).passes; }
 cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_nokey, int bits,
                       uint32_t* ka, uint32_t* kb, uint32_t* va, uint32_t* vb, uint32_t* scratch, int sms,
                       DevState* st, unsigned long long* bar_base, uint32_t* clear0, uint32_t* clear1,
-                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out, const uint32_t* plan_word,
-                      uint32_t plan_seq, bool phased) {
+                      cudaStream_t stream, uint32_t** keys_out, uint32_t** pos_out, const uint32_t* plan_keys,
+                      uint32_t* plan_word, uint32_t plan_seq, bool phased) {
   const PassPlan pl = plan_for(bits);
   if (keys_out) *keys_out = pl.passes % 2 ? ka : kb;
   if (pos_out) *pos_out = va ? (pl.passes % 2 ? va : vb) : nullptr;
   if (n == 0) return cudaSuccess;
   SortArgs a;
+  a.plan_keys = (plan_keys && plan_word && !phased) ? plan_keys : nullptr;
   a.plan_word = plan_word;
-  a.plan_seq = plan_word ? plan_seq : 0u;
+  a.plan_seq = plan_seq;
   a.phase = -1;
   a.raw = raw;
   a.n = n;
@@ -774,16 +767,6 @@ cudaError_t sort_keys(const uint32_t* raw, uint64_t n, uint64_t K, bool allow_no
   if (small)
     return va ? launch_sort<true, 4>(a, bar_base, sms, stream) : launch_sort<false, 4>(a, bar_base, sms, stream);
   return va ? launch_sort<true, kItems>(a, bar_base, sms, stream) : launch_sort<false, kItems>(a, bar_base, sms, stream);
-}
-
-void launch_plan_verify(const uint32_t* keys, const uint32_t* sk, const uint32_t* sp, uint64_t n, uint64_t K,
-                        bool allow_nokey, uint32_t seq, uint32_t* word, DevState* st, int sms, cudaStream_t stream) {
-  if (n == 0) return;
-  uint64_t b = (n + kSortThreads * 4 - 1) / (kSortThreads * 4);   // four positions per thread
-  if (b > (uint64_t)sms * 8) b = (uint64_t)sms * 8;
-  note_launches(1);
-  plan_verify_kernel<<<(unsigned)b, kSortThreads, 0, stream>>>(keys, sk, sp, n, K, allow_nokey ? 1 : 0, seq, word,
-                                                               st);
 }
 
 size_t compact_tmp_words(uint64_t n) { return (size_t)((n + kTile - 1) / kTile + 1); }

@@ -60,17 +60,42 @@ __device__ __forceinline__ const float4* row_ptr(const Store& s, const int32_t* 
                  : reinterpret_cast<const float4*>(s.main) + (uint64_t)k * D4;
 }
 
-// fixed-order block reduction of one double per thread into out[blockIdx.x]
-__device__ void block_loss(double v, double* out) {
+// Fixed-order block reduction of one double per thread into
+// o.loss_part[blockIdx.x]; with o.loss_out the last block to finish then
+// sums the partials (thread t the partials t, t + 256, ... in order, then a
+// fixed tree) into *o.loss_out and clears the block counter.
+__device__ void block_loss(double v, const StepOut& o) {
   __shared__ double sm[kThreads / 32];
+  __shared__ double tree[kThreads];
+  __shared__ int last;
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, o);
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, off);
   if ((threadIdx.x & 31) == 0) sm[threadIdx.x >> 5] = v;
   __syncthreads();
   if (threadIdx.x == 0) {
     double t = 0;
     for (int i = 0; i < kThreads / 32; ++i) t += sm[i];
-    out[blockIdx.x] = t;
+    o.loss_part[blockIdx.x] = t;
+    last = 0;
+    if (o.loss_out) {
+      __threadfence();
+      last = atomicAdd(o.loss_done, 1u) == gridDim.x - 1;
+    }
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  double t = 0.0;
+  for (unsigned i = threadIdx.x; i < gridDim.x; i += kThreads) t += __ldcg(o.loss_part + i);
+  tree[threadIdx.x] = t;
+  __syncthreads();
+  for (int w = kThreads / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) tree[threadIdx.x] += tree[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    *o.loss_out = tree[0];
+    *o.loss_done = 0u;
   }
 }
 
@@ -172,7 +197,7 @@ mf_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ rows, const uin
       o.dkeys[n + i] = kw;
     }
   }
-  block_loss(lsum, o.loss_part);
+  block_loss(lsum, o);
 }
 
 // ---------------------------------------------------------------------------
@@ -332,7 +357,7 @@ complex_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ heads, con
       o.dkeys[rrel + i] = kr;
     }
   }
-  block_loss(lsum, o.loss_part);
+  block_loss(lsum, o);
 }
 
 // ---------------------------------------------------------------------------
@@ -462,21 +487,7 @@ sgns_step_kernel(Store s, uint32_t w, const uint32_t* __restrict__ centres, cons
     }
     if (lane == 0) o.dkeys[base] = kc;
   }
-  block_loss(lsum, o.loss_part);
-}
-
-// one block: thread t sums partials t, t+256, ... in order, then a fixed tree
-__global__ void __launch_bounds__(kThreads) loss_reduce_kernel(const double* part, unsigned nparts, double* out) {
-  __shared__ double sm[kThreads];
-  double t = 0.0;
-  for (unsigned i = threadIdx.x; i < nparts; i += kThreads) t += part[i];
-  sm[threadIdx.x] = t;
-  __syncthreads();
-  for (int w = kThreads / 2; w > 0; w >>= 1) {
-    if ((int)threadIdx.x < w) sm[threadIdx.x] += sm[threadIdx.x + w];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) *out = sm[0];
+  block_loss(lsum, o);
 }
 
 }  // namespace
@@ -520,11 +531,6 @@ void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const
   else if (D4 <= 64) sgns_step_kernel<2, 4><<<grid, kThreads, 0, stream>>>(s, w, centres, contexts, negs, n, n_ctx, n_neg, vocab, lr, o);
   else if (D4 <= 96) sgns_step_kernel<3, 2><<<grid, kThreads, 0, stream>>>(s, w, centres, contexts, negs, n, n_ctx, n_neg, vocab, lr, o);
   else sgns_step_kernel<8, 1><<<grid, kThreads, 0, stream>>>(s, w, centres, contexts, negs, n, n_ctx, n_neg, vocab, lr, o);
-}
-
-void launch_loss_reduce(const double* part, unsigned nparts, double* out, cudaStream_t stream) {
-  note_launches(1);
-  loss_reduce_kernel<<<1, kThreads, 0, stream>>>(part, nparts, out);
 }
 
 }  // namespace adapm

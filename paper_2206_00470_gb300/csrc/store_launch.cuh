@@ -95,6 +95,8 @@ struct StepOut {
   float* drows;
   double* loss_part;     // grid-sized partial sums
   unsigned loss_blocks;  // number of partials written
+  double* loss_out;      // the batch loss (summed by the last block), or nullptr
+  uint32_t* loss_done;   // blocks finished (zero between launches)
 };
 
 void launch_mf_step(const Store& s, uint32_t w, const uint32_t* rows, const uint32_t* cols,
@@ -109,6 +111,5 @@ void launch_sgns_step(const Store& s, uint32_t w, const uint32_t* centres, const
                       uint32_t vocab, uint32_t dim, float lr, const StepOut& o, int sms,
                       cudaStream_t stream);
 unsigned step_loss_blocks(int sms);
-void launch_loss_reduce(const double* part, unsigned nparts, double* out, cudaStream_t stream);
 
 }  // namespace adapm

@@ -225,3 +225,34 @@ def test_complex_step_uses_its_plan(gpu_lib):
     main = pm.read_main(np.arange(cfg.num_keys))
     assert np.max(np.abs(main - ref.main)) <= 1e-5 * np.abs(ref.main).max()
     pm.close()
+
+
+def test_step_with_other_keys_misses_its_plan(gpu_lib):
+    """A training step compares the push keys it writes with its plan's keys: a step on another batch of the
+    same size counts one miss, sorts its keys, and gives the bits a run without plans gives."""
+    cfg = dataclasses.replace(wl.MF, name="mf_small", rows=5000, cols=800, rank=8, workers=1, batch=1500,
+                              lookahead=1, zipf_s=1.1, total_cells=10 ** 6)
+    init = init_rows_np(np.arange(cfg.num_keys), cfg.value_len, cfg.rank, cfg.seed, cfg.init_std)
+    a = [x.cuda() for x in wl.mf_batch(cfg, 0, 1)]
+    b = [x.cuda() for x in wl.mf_batch(cfg, 0, 2)]
+    out, losses = [], []
+    for plans in (True, False):
+        pm = gpu_lib.ParameterManager(cfg.num_keys, cfg.value_len, 1, init_values=torch.from_numpy(init).cuda(),
+                                      push_plans=plans)
+        pm.intent(0, torch.cat(a[:2]), 1, 3)     # signals batch a ...
+        pm.advance_clock(0)
+        loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+        pm.mf_step(0, b[0], b[1], b[2], cfg.rank, True, cfg.lr, cfg.eps, loss_out=loss)   # ... trains on b
+        pm.mf_step(0, a[0], a[1], a[2], cfg.rank, True, cfg.lr, cfg.eps)                  # then on a
+        pm.advance_clock(0)
+        pm.advance_clock(0)
+        pm.wait()
+        out.append(pm.read_main(np.arange(cfg.num_keys)))
+        losses.append(float(loss.item()))
+        st = pm.stats()
+        if plans:
+            assert st["planned_pushes"] == 2 and st["plan_misses"] == 1
+        else:
+            assert st["planned_pushes"] == 0
+        pm.close()
+    assert np.array_equal(out[0], out[1]) and losses[0] == losses[1]
