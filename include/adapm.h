@@ -347,6 +347,14 @@ const char* adapm_last_error(adapm_ctx* ctx);
  * other contexts are unaffected. */
 adapm_status adapm_debug_fail_next_barrier(adapm_ctx* ctx);
 
+/* Fault injection for tests of CUDA error handling (no GPU fault is
+ * involved, nothing on the device changes): the next call of this context
+ * that launches kernels enqueues them and then returns ADAPM_ECUDA as if
+ * the CUDA runtime had reported a launch failure.  As after a real one, the
+ * context is unusable afterwards (every later call returns ADAPM_ECUDA);
+ * other contexts are unaffected. */
+adapm_status adapm_debug_fail_next_launch(adapm_ctx* ctx);
+
 #ifdef __cplusplus
 }
 #endif

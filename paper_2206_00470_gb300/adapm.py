@@ -27,7 +27,7 @@ EXPORTS = [
     "adapm_sgns_step", "adapm_clock", "adapm_replica_keys", "adapm_replica_rows",
     "adapm_refcounts", "adapm_owners", "adapm_poisson_quantile", "adapm_read_main", "adapm_get_stats", "adapm_profile_enable",
     "adapm_profile_read", "adapm_kernel_launches", "adapm_push_noalloc", "adapm_last_error",
-    "adapm_debug_fail_next_barrier",
+    "adapm_debug_fail_next_barrier", "adapm_debug_fail_next_launch",
 ]
 
 
@@ -119,6 +119,7 @@ def load(path=LIB_PATH):
         "adapm_kernel_launches": [ctypes.POINTER(U64)],
         "adapm_push_noalloc": [P, U32, P, U64, P],
         "adapm_debug_fail_next_barrier": [P],
+        "adapm_debug_fail_next_launch": [P],
     }
     for name, args in sig.items():
         fn = getattr(L, name)
@@ -304,6 +305,10 @@ class ParameterManager:
     def debug_fail_next_barrier(self):
         """Test hook: the next push's sort gives up its grid-barrier wait (ADAPM_ETIMEOUT at wait)."""
         self._check(self._lib.adapm_debug_fail_next_barrier(self._h))
+
+    def debug_fail_next_launch(self):
+        """Test hook: the next call that launches kernels returns ADAPM_ECUDA as after a launch failure."""
+        self._check(self._lib.adapm_debug_fail_next_launch(self._h))
 
     def sync(self):
         self._check(self._lib.adapm_sync(self._h))

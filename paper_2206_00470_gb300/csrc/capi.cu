@@ -124,6 +124,7 @@ struct adapm_ctx {
   AdvCounts* early_counts = nullptr;
   uint64_t early_advances = 0;   // advances that used their early events
   uint64_t early_undone = 0;     // early events taken back
+  bool fake_launch_error = false;   // adapm_debug_fail_next_launch
 };
 
 namespace {
@@ -369,6 +370,8 @@ struct ProfScope {
 
 adapm_status check_launch(adapm_ctx* ctx, const char* where) {
   cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && ctx->fake_launch_error) e = cudaErrorLaunchFailure;   // adapm_debug_fail_next_launch
+  ctx->fake_launch_error = false;
   if (e != cudaSuccess) return cuda_fail(ctx, e, where);
   return ADAPM_OK;
 }
@@ -706,6 +709,13 @@ void adapm::ctx_add_push_rows(adapm_ctx* ctx, uint64_t n) {
 int adapm::ctx_begin(adapm_ctx* ctx) { return check_ctx(ctx); }
 
 int adapm::ctx_fail_cuda(adapm_ctx* ctx, cudaError_t e, const char* where) { return cuda_fail(ctx, e, where); }
+
+cudaError_t adapm::ctx_launch_error(adapm_ctx* ctx) {
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && ctx->fake_launch_error) e = cudaErrorLaunchFailure;   // adapm_debug_fail_next_launch
+  ctx->fake_launch_error = false;
+  return e;
+}
 
 ProfToken adapm::ctx_prof_start(adapm_ctx* ctx, int op) {
   ProfToken t;
@@ -1055,6 +1065,12 @@ adapm_status adapm_sync(adapm_ctx* ctx) {
 adapm_status adapm_poisson_quantile(double lambda, double p, int64_t* out) {
   if (!out || !(lambda > 0.0) || !(p > 0.0 && p < 1.0)) return ADAPM_EINVAL;
   *out = poisson_quantile(lambda, p);
+  return ADAPM_OK;
+}
+
+adapm_status adapm_debug_fail_next_launch(adapm_ctx* ctx) {
+  if (!ctx) return ADAPM_EINVAL;
+  ctx->fake_launch_error = true;
   return ADAPM_OK;
 }
 

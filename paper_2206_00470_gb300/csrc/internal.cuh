@@ -186,6 +186,9 @@ int ctx_begin(struct ::adapm_ctx* ctx);
 // A CUDA runtime error: records "where: message", marks the context unusable
 // (as every entry point does) and returns ADAPM_ECUDA.
 int ctx_fail_cuda(struct ::adapm_ctx* ctx, cudaError_t e, const char* where);
+// cudaGetLastError() after a call's launches, or the launch failure that
+// adapm_debug_fail_next_launch asked for (taken once).
+cudaError_t ctx_launch_error(struct ::adapm_ctx* ctx);
 // Per-operation timing (adapm_profile_enable): events recorded around an
 // operation's work on the context's stream; a no-op while profiling is off.
 struct ProfToken {

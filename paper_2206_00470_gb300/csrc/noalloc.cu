@@ -153,7 +153,7 @@ extern "C" adapm_status adapm_push_noalloc(adapm_ctx* ctx, uint32_t worker, cons
     ProfGuard scatter(ctx, 6);
     launch_push(v.s, a, v.sms, v.stream);
   }
-  e = cudaGetLastError();
+  e = ctx_launch_error(ctx);
   if (e != cudaSuccess) return static_cast<adapm_status>(ctx_fail_cuda(ctx, e, "push_noalloc scatter"));
   return ADAPM_OK;
 }

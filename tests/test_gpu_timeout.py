@@ -46,3 +46,34 @@ def test_barrier_wait_gives_up_and_leaves_the_store(gpu_lib):
     pm2.wait()
     assert np.array_equal(pm2.read_main(np.arange(K)), before)
     pm2.close()
+
+
+@pytest.mark.parametrize("call", ["push", "push_noalloc", "pull"])
+def test_launch_failure_retires_the_context(gpu_lib, call):
+    """A CUDA error after a call's launches (injected on the host: no GPU fault) retires the context, for the
+    allocation-free push as for every other entry point; later calls report it and other contexts work."""
+    A = gpu_lib
+    K, D = 500, 8
+    pm = A.ParameterManager(K, D, 1)
+    keys = torch.arange(0, 64, device="cuda", dtype=torch.int32)
+    deltas = torch.ones(64, D, device="cuda")
+    pm.push(0, keys, deltas)
+    pm.wait()
+    pm.debug_fail_next_launch()
+    with pytest.raises(A.AdaPMError) as e:
+        if call == "pull":
+            pm.pull(0, keys)
+        else:
+            getattr(pm, call)(0, keys, deltas)
+    assert e.value.status == A.ECUDA
+    assert pm.last_error() != ""
+    for retry in (lambda: pm.push(0, keys, deltas), lambda: pm.push_noalloc(0, keys, deltas), pm.wait):
+        with pytest.raises(A.AdaPMError) as e:
+            retry()
+        assert e.value.status == A.ECUDA
+    pm.close()
+    pm2 = A.ParameterManager(K, D, 1)
+    pm2.push_noalloc(0, keys, deltas)
+    pm2.wait()
+    assert np.array_equal(pm2.read_main(np.arange(64)), np.ones((64, D), np.float32))
+    pm2.close()
