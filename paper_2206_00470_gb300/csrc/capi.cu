@@ -531,8 +531,10 @@ IntentList* find_plan(adapm_ctx* ctx, uint32_t w, uint64_t n) {
   return nullptr;
 }
 
+// plans = false: the caller knows its keys never follow an intent's order
+// (the SGNS step), so no plan is looked up.
 adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint64_t n,
-                         const float* drows, bool allow_nokey) {
+                         const float* drows, bool allow_nokey, bool plans = true) {
   if (n == 0) return ADAPM_OK;
   {
     const adapm_status st = early_make(ctx, w);
@@ -543,7 +545,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   // keys are the ones the plan was made from, and sorts (into this push's
   // own arrays) only if they are not; the scatter kernels read the plan's
   // arrays or the sort's by the same check
-  IntentList* plan = find_plan(ctx, w, n);
+  IntentList* plan = plans ? find_plan(ctx, w, n) : nullptr;
   uint32_t seq = 0;
   if (plan) {
     CK(cudaStreamWaitEvent(ctx->stream, plan->ready, 0));
@@ -1253,7 +1255,9 @@ adapm_status adapm_sgns_step(adapm_ctx* ctx, uint32_t worker, const uint32_t* ce
   }
   {
     ProfScope ps(ctx, 3);
-    st = push_device(ctx, worker, o.dkeys, m, o.drows, true);
+    // its rows follow the centres (each with its context and negative slots),
+    // never an intent's key order: no plan
+    st = push_device(ctx, worker, o.dkeys, m, o.drows, true, /*plans=*/false);
   }
   if (loss_out) CK(finish_out(ctx, &lo));
   for (void* p : {(void*)ic.owned, (void*)ix.owned, (void*)ineg.owned, (void*)o.dkeys,

@@ -671,7 +671,10 @@ cudaError_t launch_sort(SortArgs& a, unsigned long long* bar_base, int sms, cuda
   constexpr uint64_t SUB = (uint64_t)kSortThreads * ITEMS;
   const int occ = sort_blocks_per_sm<POS, ITEMS>();
   uint64_t B = (a.n + SUB - 1) / SUB;
-  const uint64_t resident = (uint64_t)sms * (occ < 4 ? occ : 4);
+  // A launch that checks a plan expects it to match and only to check: one
+  // block per SM needs room for one block on each SM, not four, before it can
+  // start beside other streams' kernels (a miss then sorts with that grid).
+  const uint64_t resident = (uint64_t)sms * (a.plan_keys ? 1 : (occ < 4 ? occ : 4));
   if (B > resident) B = resident;
   if (B > kMaxSortBlocks) B = kMaxSortBlocks;
   if (B < 1) B = 1;

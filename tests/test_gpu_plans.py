@@ -256,3 +256,22 @@ def test_step_with_other_keys_misses_its_plan(gpu_lib):
             assert st["planned_pushes"] == 0
         pm.close()
     assert np.array_equal(out[0], out[1]) and losses[0] == losses[1]
+
+
+def test_sgns_step_sorts_without_a_plan(gpu_lib):
+    """The SGNS step's rows follow its centres, never an intent's key order: it looks up no plan, even when an
+    intent of exactly its push's size is active, and sorts."""
+    vocab, dim, n, n_ctx, n_neg = 300, 16, 40, 4, 3
+    K = 2 * vocab
+    rng = np.random.default_rng(5)
+    pm = gpu_lib.ParameterManager(K, dim, 1)
+    centres = torch.as_tensor(rng.integers(0, vocab, size=n), dtype=torch.int32, device="cuda")
+    contexts = torch.as_tensor(rng.integers(0, vocab, size=n * n_ctx), dtype=torch.int32, device="cuda")
+    negatives = torch.as_tensor(rng.integers(0, vocab, size=n * n_ctx * n_neg), dtype=torch.int32, device="cuda")
+    m = n * (1 + n_ctx * (1 + n_neg))
+    pm.intent(0, torch.as_tensor(rng.integers(0, K, size=m), device="cuda"), 0, 2)
+    pm.sgns_step(0, centres, contexts, negatives, n_ctx, n_neg, vocab, dim, 0.05)
+    pm.wait()
+    st = pm.stats()
+    assert st["planned_pushes"] == 0 and st["plan_misses"] == 0 and st["push_rows"] == m
+    pm.close()
