@@ -98,6 +98,8 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : (VER && C == 1 ? 3 : 4)
   float4* acc4 = reinterpret_cast<float4*>(s.acc);
   const uint64_t g = group_id<G>(), ng = group_count<G>();
   uint32_t nkeys = 0, nreps = 0, nref = 0;   // nref: VER only
+  __shared__ int32_t hslots[kThreads / G][32];   // holders' slots of the key a group merges (W <= 32)
+  const unsigned gmask = G == 32 ? 0xFFFFFFFFu : (((1u << G) - 1u) << ((threadIdx.x & 31) & ~(G - 1)));
   // R slots per group at a time: owners, holder masks, then (for keys held
   // by one worker only, the common case) main and pending rows, each as one
   // round of independent loads.  Versioned refresh (App. B.1.2: a holder
@@ -168,58 +170,121 @@ __global__ void __launch_bounds__(kThreads, C >= 8 ? 2 : (VER && C == 1 ? 3 : 4)
           s.dirty[k] = 0;
         }
       }
-      float4 m[C];
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
-      }
-      constexpr int Q = 4 / C > 0 ? 4 / C : 1;
-      uint32_t mm = mask;
-      while (mm) {
-        int32_t hs[Q];
-#pragma unroll
-        for (int q = 0; q < Q; ++q) {
-          hs[q] = -1;
-          if (mm) {
-            const uint32_t wb = __ffs(mm) - 1;
-            mm &= mm - 1;
-            hs[q] = s.map[(uint64_t)wb * s.K + k];
-          }
-        }
-        float4 t[Q][C];
-#pragma unroll
-        for (int q = 0; q < Q; ++q)
-#pragma unroll
-          for (int c = 0; c < C; ++c) {
-            const uint32_t col = lane + c * G;
-            t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
-          }
-#pragma unroll
-        for (int q = 0; q < Q; ++q)
-          if (hs[q] >= 0)
-#pragma unroll
-            for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
-      }
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const uint32_t col = lane + c * G;
-        if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
-      }
-      mm = mask;
-      while (mm) {
-        const uint32_t wb = __ffs(mm) - 1;
-        mm &= mm - 1;
-        const int32_t h = s.map[(uint64_t)wb * s.K + k];
-        if (h < 0) continue;
+      // Holders that fit in one round of Q rows: their slots are looked up with
+      // the sum and again for the writes.  More: each lane looks up one
+      // holder's slot (G at a time) into shared memory, so the sum and the
+      // writes need no second lookup.  Both add the pending rows to main in
+      // ascending worker order.
+      if (__popc(mask) <= (4 / C > 0 ? 4 / C : 1)) {
+        float4 m[C];
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const uint32_t col = lane + c * G;
-          if (col < D4) {
-            val4[(uint64_t)h * D4 + col] = m[c];
-            acc4[(uint64_t)h * D4 + col] = f4zero();
+          m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
+        }
+        constexpr int Q = 4 / C > 0 ? 4 / C : 1;
+        uint32_t mm = mask;
+        while (mm) {
+          int32_t hs[Q];
+#pragma unroll
+          for (int q = 0; q < Q; ++q) {
+            hs[q] = -1;
+            if (mm) {
+              const uint32_t wb = __ffs(mm) - 1;
+              mm &= mm - 1;
+              hs[q] = s.map[(uint64_t)wb * s.K + k];
+            }
+          }
+          float4 t[Q][C];
+#pragma unroll
+          for (int q = 0; q < Q; ++q)
+#pragma unroll
+            for (int c = 0; c < C; ++c) {
+              const uint32_t col = lane + c * G;
+              t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
+            }
+#pragma unroll
+          for (int q = 0; q < Q; ++q)
+            if (hs[q] >= 0)
+#pragma unroll
+              for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
+        }
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
+        }
+        mm = mask;
+        while (mm) {
+          const uint32_t wb = __ffs(mm) - 1;
+          mm &= mm - 1;
+          const int32_t h = s.map[(uint64_t)wb * s.K + k];
+          if (h < 0) continue;
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            if (col < D4) {
+              val4[(uint64_t)h * D4 + col] = m[c];
+              acc4[(uint64_t)h * D4 + col] = f4zero();
+            }
           }
         }
+      } else {
+        float4 m[C];   // (loaded with the holders' slots)
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          m[c] = col < D4 ? main4[(uint64_t)k * D4 + col] : f4zero();
+        }
+        // the holders' slots: one slot-map lookup per lane (holder j by lane j,
+        // G at a time), kept in shared memory for the sum and the writes
+        const int nh = __popc(mask);
+        int32_t* hsl = hslots[threadIdx.x / G];
+        for (int j = lane; j < nh; j += G) {
+          uint32_t mm = mask;   // the j-th set bit (j < nh, so mm stays nonzero)
+          for (int t = 0; t < j; ++t) mm &= mm - 1;
+          const uint32_t wb = (uint32_t)(__ffs(mm) - 1);
+          hsl[j] = s.map[(uint64_t)wb * s.K + k];
+        }
+        __syncwarp(gmask);
+        constexpr int Q = 4 / C > 0 ? 4 / C : 1;
+        // pending rows added in ascending worker order, Q rows in flight
+        for (int j0 = 0; j0 < nh; j0 += Q) {
+          int32_t hs[Q];
+#pragma unroll
+          for (int q = 0; q < Q; ++q) hs[q] = j0 + q < nh ? hsl[j0 + q] : -1;
+          float4 t[Q][C];
+#pragma unroll
+          for (int q = 0; q < Q; ++q)
+#pragma unroll
+            for (int c = 0; c < C; ++c) {
+              const uint32_t col = lane + c * G;
+              t[q][c] = (hs[q] >= 0 && col < D4) ? acc4[(uint64_t)hs[q] * D4 + col] : f4zero();
+            }
+#pragma unroll
+          for (int q = 0; q < Q; ++q)
+            if (hs[q] >= 0)
+#pragma unroll
+              for (int c = 0; c < C; ++c) m[c] = f4add(m[c], t[q][c]);
+        }
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const uint32_t col = lane + c * G;
+          if (col < D4) main4[(uint64_t)k * D4 + col] = m[c];
+        }
+        for (int j = 0; j < nh; ++j) {
+          const int32_t h = hsl[j];
+          if (h < 0) continue;
+#pragma unroll
+          for (int c = 0; c < C; ++c) {
+            const uint32_t col = lane + c * G;
+            if (col < D4) {
+              val4[(uint64_t)h * D4 + col] = m[c];
+              acc4[(uint64_t)h * D4 + col] = f4zero();
+            }
+          }
+        }
+        __syncwarp(gmask);   // hsl is reused by the group's next key
       }
     }
   }
