@@ -226,3 +226,26 @@ def test_host_intent_keys_with_early_events(gpu_lib, host):
     assert pm.stats()["early_advances"] > 0
     compare_full_state(pm, ref, K, W)
     pm.close()
+
+
+def test_allocation_free_push_between_early_events_and_the_advance(gpu_lib):
+    """The allocation-free push makes no early events of its own (it allocates nothing); the pull before it
+    does, and the advance uses them: the same state as the oracle."""
+    K, D, W = 2000, 32, 3
+    init = dyadic_init(K, D, 23)
+    ops = loop_ops(31, K, D, W, 5, 500, 1, 1)
+    pm = gpu_lib.ParameterManager(K, D, W, init_values=torch.from_numpy(init).cuda())
+    ref = ParameterManagerOracle(K, D, W, init)
+    for op in ops:
+        if op["op"] == "push":
+            pm.push_noalloc(op["w"], dev(op["keys"]), torch.from_numpy(np.ascontiguousarray(op["deltas"])).cuda())
+        else:
+            got = apply_gpu(pm, op)
+            if op["op"] == "pull":
+                assert np.array_equal(got, ref.pull(op["w"], op["keys"]))
+                continue
+        apply_ref(ref, op)
+    st = pm.stats()
+    assert st["early_advances"] == 5 * W and st["early_undone"] == 0
+    compare_full_state(pm, ref, K, W)
+    pm.close()
