@@ -156,7 +156,9 @@ adapm_status adapm_destroy(adapm_ctx* ctx);
  * device that its keys equal that intent's, position by position, and then
  * groups its rows by the stored sort instead of sorting again; otherwise it
  * sorts.  Results are the same either way (the same stable order).  The SGNS
- * step, whose rows never follow an intent's key order, always sorts.
+ * step, whose rows never follow an intent's key order, always sorts.  A
+ * worker whose last four plans went unused gets plans for one intent in
+ * sixteen only, until a push takes one again.
  * adapm_wait also waits for that stream. */
 adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys, uint64_t n,
                           int64_t clock_start, int64_t clock_end);

@@ -44,6 +44,7 @@ struct IntentList {
   uint32_t* px = nullptr;     // the call's keys as given (what a matching push's keys equal)
   uint64_t n = 0;
   bool from_plan = false;
+  bool plan_used = false;      // a push took this plan
   cudaEvent_t ready = nullptr;
   void* in_owned = nullptr;   // the call's staged copy of host keys, read by the plan stream
   int64_t start = 0, end = 0; // the window as signalled
@@ -56,6 +57,11 @@ struct WorkerState {
   std::map<int64_t, std::vector<int64_t>> starts;   // clock -> lists whose window opens
   std::map<int64_t, std::vector<int64_t>> ends;     // clock -> lists whose window closes
   std::vector<int64_t> order;                       // recorded lists, oldest first
+  // Lists closed in a row whose plan no push took, and intents recorded: a
+  // worker whose pushes never match its intents (the SGNS step) stops
+  // getting plans, except every kPlanProbe-th intent.
+  int unused_plans = 0;
+  uint64_t intents = 0;
   // Early events of the next advance (made at the worker's first push after
   // its last advance): the lists they cover, the create and evict lists
   // they fill, and the event after them on the early stream.
@@ -385,6 +391,8 @@ adapm_status check_ctx(adapm_ctx* ctx) {
 }
 
 constexpr uint64_t kMaxN = 1ull << 31;
+constexpr int kPlanPatience = 4;       // unused plans in a row after which a worker gets none ...
+constexpr uint64_t kPlanProbe = 16;    // ... but for one intent in this many
 
 // Refcount events of one worker -> destroy, then create replicas.
 // ---------------------------------------------------------------------------
@@ -548,6 +556,7 @@ adapm_status push_device(adapm_ctx* ctx, uint32_t w, const uint32_t* dkeys, uint
   IntentList* plan = plans ? find_plan(ctx, w, n) : nullptr;
   uint32_t seq = 0;
   if (plan) {
+    plan->plan_used = true;
     CK(cudaStreamWaitEvent(ctx->stream, plan->ready, 0));
     if (++ctx->plan_seq == 0) ctx->plan_seq = 1;
     seq = ctx->plan_seq;
@@ -674,6 +683,10 @@ cudaError_t make_plan(adapm_ctx* ctx, IntentList& L, const uint32_t* keys, cudaE
 cudaError_t close_list(adapm_ctx* ctx, uint32_t w, int64_t id) {
   IntentList& L = ctx->lists[id];
   cudaError_t e = cudaSuccess;
+  if (L.psk) {
+    int& unused = ctx->workers[w].unused_plans;
+    unused = L.plan_used ? 0 : unused + 1;
+  }
   if (L.ready) {
     e = cudaStreamWaitEvent(ctx->stream, L.ready, 0);
     ctx->spare_ready.push_back(L.ready);   // the wait has captured it; it can be recorded again
@@ -895,7 +908,10 @@ adapm_status adapm_intent(adapm_ctx* ctx, uint32_t worker, const uint32_t* keys,
   L.start = signalled_start;
   L.end = clock_end;
   const bool now = clock_start <= ws.clock;   // the window contains the current clock: active at once
-  const bool plan = n > 0 && !ctx->cfg.no_push_plans;
+  // a plan unless the worker's recent ones all went unused (then one probe in kPlanProbe)
+  const bool plan = n > 0 && !ctx->cfg.no_push_plans &&
+                    (ws.unused_plans < kPlanPatience || ws.intents % kPlanProbe == 0);
+  ws.intents += 1;
   CK(cudaMallocFromPoolAsync((void**)&L.keys, (n + 1) * sizeof(uint32_t), ctx->pool, ctx->stream));
   L.count = L.keys + n;
   if (n == 0) {

@@ -275,3 +275,33 @@ def test_sgns_step_sorts_without_a_plan(gpu_lib):
     st = pm.stats()
     assert st["planned_pushes"] == 0 and st["plan_misses"] == 0 and st["push_rows"] == m
     pm.close()
+
+
+def test_worker_whose_plans_go_unused_stops_getting_them(gpu_lib):
+    """After four lists in a row closed with a plan no push took, a worker's intents get no plan, except one
+    intent in sixteen (a probe); a probe that a push takes brings plans back.  Results match the oracle."""
+    K, D, n = 3000, 8, 400
+    rng = np.random.default_rng(21)
+    init = dyadic_init(K, D, 8)
+    pm = gpu_lib.ParameterManager(K, D, 1, init_values=torch.from_numpy(init).cuda())
+    ref = ParameterManagerOracle(K, D, 1, init)
+    planned = []
+    for c in range(20):   # intents 0..19 (clock c signals clock c + 1); intent 16 is a probe
+        keys = hot_keys(rng, K, n)
+        for api, cv in ((pm, lambda x: torch.as_tensor(x, device="cuda")), (ref, lambda x: x)):
+            api.intent(0, cv(keys), c + 1, c + 2)
+            api.advance_clock(0)
+        # clocks 1..15 push other keys (the plan goes unused); from clock 17 the signalled ones
+        push = keys if c >= 16 else hot_keys(rng, K, n // 2)
+        d = dyadic_rows(rng, len(push), D)
+        pm.push(0, torch.as_tensor(push, device="cuda"), torch.from_numpy(d).cuda())
+        ref.push(0, push, d)
+        pm.wait()
+        planned.append(pm.stats()["planned_pushes"])
+    check_same(pm, ref, K, 1)
+    # intents 5..15 were recorded after 4 or more unused plans: none has a plan; intent 16 is a probe and the
+    # push of clock 17 takes it
+    assert planned[15] == 0 and planned[16] == 1
+    # intent 17 was recorded before the probe's list closed (no plan); 18 and 19 have plans again
+    assert planned[17] == 1 and planned[18] == 2 and planned[19] == 3
+    pm.close()
