@@ -74,3 +74,21 @@ def test_source_digest_ignores_comments(tmp_path):
     assert bench.source_digest([str(a)]) == bench.source_digest([str(b)])
     b.write_text("int x = 1;\nint y = 3;\n")
     assert bench.source_digest([str(a)]) != bench.source_digest([str(b)])
+
+
+def test_manager_options_name_every_switch():
+    """The `config` of a bench line names the manager's options, the flags turn them off or on, and the
+    microbenchmark record keeps them."""
+    on = argparse.Namespace(relocate=False, timing="start", delta_refresh=False, no_push_plans=False,
+                            pull_staging=False, no_early_events=False)
+    off = argparse.Namespace(relocate=True, timing="adaptive", delta_refresh=True, no_push_plans=True,
+                             pull_staging=True, no_early_events=True)
+    a, b = bench.manager_options(on), bench.manager_options(off)
+    assert a["push_plans"] and a["early_events"] and a["placement"] == "replicate" and a["refresh"] == "full"
+    assert not b["push_plans"] and not b["early_events"] and b["placement"] == "relocate"
+    assert b["action_timing"] == "adaptive" and b["refresh"] == "versioned" and b["pull"] != a["pull"]
+    m = bench.micro_args(argparse.Namespace(workload="mf", batch=4, zipf=None, span=2, keys=7, steps=3,
+                                            no_early_events=True), 1.4)
+    assert m.workload == "micro" and m.zipf == 1.4 and m.batch is None and m.keys is None and m.span is None
+    assert m.no_early_events and m.steps == 3
+    assert "early_events_per_step" in bench.MICRO_KEYS and "early_advances" in bench.COUNTERS
